@@ -1,0 +1,401 @@
+"""Benchmark: ragged causal GQA prefill attention on GB300 (libopattn).
+
+One step = one pass of the whole hot path (one persistent-kernel launch of
+opattn over the workload's ragged batch).  The headline workload is the
+Llama-3-70B-shaped layer (Hq 64, Hkv 8, d 128, 8 prompts x 4096 tokens).
+
+Metric: causal attention TFLOP/s, counting 4 * d * Hq FLOPs per visible
+(query, key) pair (2d for QK^T, 2d for PV; masked and skipped work, softmax
+and the dense square are not counted); tokens/s and the fraction of the
+measured dense BF16 peak are printed beside it.
+
+Arms:
+  --impl ours       (default) the CUDA library; `value` is kernel time with
+                    inputs resident in HBM, `e2e` goes through the C-ABI
+                    one-shot call with pinned host buffers and includes the
+                    host<->device copies.
+  --impl reference  the fp64 CPU oracle on this machine's cores, each step a
+                    bounded row sample of the same workload.
+
+Multi-GPU (torchrun, one process per GPU): every rank runs an independent
+replica of the workload (the operator shards by sequence or kv head with no
+data exchange); timing is the max over ranks, value the sum of all ranks'
+work over that time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "prefill attention TFLOP/s (causal) and prompt tokens/s on 1 GB300; % BF16 peak"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ---------------------------------------------------------------- helpers
+
+def visible_pairs(q_lens, k_lens) -> int:
+    """Number of (query, key) pairs the bottom-right causal mask leaves visible."""
+    total = 0
+    for lq, lk in zip(q_lens, k_lens):
+        if lq == 0 or lk == 0:
+            continue
+        i = np.arange(lq, dtype=np.int64)
+        total += int(np.clip(i + (lk - lq) + 1, 0, lk).sum())
+    return total
+
+
+def causal_flops(w) -> int:
+    return 4 * w.d * w.Hq * visible_pairs(w.q_lens, w.k_lens)
+
+
+def row_flops(w, tokens, heads) -> int:
+    """Causal FLOPs of selected output rows (same per-pair count)."""
+    seq = np.searchsorted(w.cu_q, tokens, side="right") - 1
+    lq = np.asarray(w.q_lens)[seq]
+    lk = np.asarray(w.k_lens)[seq]
+    i = tokens - w.cu_q[seq]
+    n = np.clip(i + (lk - lq) + 1, 0, lk)
+    return int(4 * w.d * n.sum())
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def aggregate_over_ranks(elapsed_s: float, work_units: float, dist=None):
+    """(max elapsed over ranks, sum of work over ranks); identity without a process group."""
+    if dist is None or not dist.is_available() or not dist.is_initialized():
+        return elapsed_s, work_units
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([elapsed_s], dtype=torch.float64, device=dev)
+    u = torch.tensor([work_units], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+    def __init__(self, gpu_selector: str | None):
+        self.sel = gpu_selector
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if self.sel:
+            cmd += ["-i", self.sel]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(self.NAMES, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm), "sm_mhz_min": min(sm)}
+
+
+def gpu_selector(torch, dev):
+    props = torch.cuda.get_device_properties(dev)
+    uuid = getattr(props, "uuid", None)
+    if uuid:
+        s = str(uuid)
+        return s if s.startswith("GPU-") else "GPU-" + s
+    return str(dev)
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name"):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return "unknown"
+
+
+def oracle_sample(w, q, k, v, seconds: float, seed: int = 0):
+    """Time the fp64 oracle on random rows of w for about `seconds`; returns a dict."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    threads = oracle.default_threads()
+    n = max(8, threads)
+    done_flops, done_rows, t_total = 0, 0, 0.0
+    while t_total < seconds:
+        tok = rng.integers(0, w.total_q, size=n).astype(np.int64)
+        hd = rng.integers(0, w.Hq, size=n).astype(np.int32)
+        t0 = time.perf_counter()
+        oracle.attention_rows(q, k, v, w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale, tok, hd, n_threads=threads)
+        dt = time.perf_counter() - t0
+        t_total += dt
+        done_flops += row_flops(w, tok, hd)
+        done_rows += n
+        if dt < seconds / 8:
+            n *= 2
+    return {"flops": done_flops, "seconds": t_total, "rows": done_rows, "threads": threads}
+
+
+# ----------------------------------------------------------- reference arm
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import torch
+    from paper_2608_13499_gb300 import workloads as W
+    q, k, v = W.make_inputs(w, "cpu")
+    qb, kb, vb = q, k, v
+    per_step = max(0.5, args.reference_step_seconds)
+    for _ in range(args.warmup):
+        oracle_sample(w, qb, kb, vb, per_step / 4, seed=1)
+    flops, secs, rows = 0, 0.0, 0
+    for s in range(args.steps):
+        r = oracle_sample(w, qb, kb, vb, per_step, seed=100 + s)
+        flops += r["flops"]
+        secs += r["seconds"]
+        rows += r["rows"]
+        threads = r["threads"]
+    value = flops / secs / 1e12
+    tokens_per_s = value * 1e12 / (causal_flops(w) / w.total_q)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded N(0,1) bf16 inputs; counter-based generator)",
+        "config": dict(w.describe(), sample="random (token, head) rows per step"),
+        "tokens_per_s": tokens_per_s,
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
+                         "sample": f"{rows} random output rows of {w.name} over {args.steps} steps, "
+                                   f"~{per_step:.1f} s each, fp64, {cpu_model()}"},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# -------------------------------------------------------------- our arm
+
+def run_ours(args, w):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_13499_gb300 as pkg
+    from paper_2608_13499_gb300 import build as pbuild
+    from paper_2608_13499_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={world}: launch N>1 with torchrun")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or world == 1:
+        pbuild.build()
+    if world > 1:
+        dist.barrier()
+    pkg.load()
+
+    peaks, peak_src = load_peaks()
+    q, k, v = W.make_inputs(w, dev)
+    o = torch.empty((w.total_q, w.Hq, w.d), dtype=torch.bfloat16, device=dev)
+    lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device=dev)
+    flops = causal_flops(w)
+    stream = torch.cuda.current_stream(dev)
+
+    plan = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d)
+    for _ in range(max(args.warmup, 3)):
+        plan.run(q, k, v, o, lse, w.scale, stream)
+    torch.cuda.synchronize(dev)
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    sampler = ClockSampler(gpu_selector(torch, local))
+    sampler.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        plan.run(q, k, v, o, lse, w.scale, stream)
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    elapsed = t_start.elapsed_time(t_end) / 1e3
+    launch_ms = [a.elapsed_time(b) for a, b in ev]
+    elapsed_max, flops_all = aggregate_over_ranks(elapsed, float(flops) * args.steps, dist if world > 1 else None)
+    value = flops_all / elapsed_max / 1e12
+    kernel_ms = statistics.mean(launch_ms)
+    achieved = flops / (kernel_ms / 1e3) / 1e12
+
+    # end to end through the one-shot C-ABI call with pinned host buffers
+    e2e_steps = max(3, min(args.steps, args.e2e_steps))
+    hq = q.cpu().pin_memory()
+    hk = k.cpu().pin_memory()
+    hv = v.cpu().pin_memory()
+    ho = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    hl = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+
+    def e2e_step():
+        dq.copy_(hq, non_blocking=True)
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
+        pkg.opattn_prefill(dq, dk, dv, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
+        ho.copy_(o, non_blocking=True)
+        hl.copy_(lse, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_elapsed, e2e_flops = aggregate_over_ranks(e0.elapsed_time(e1) / 1e3, float(flops) * e2e_steps,
+                                                  dist if world > 1 else None)
+    e2e_value = e2e_flops / e2e_elapsed / 1e12
+    h2d = q.numel() * 2 + k.numel() * 2 + v.numel() * 2
+    d2h = o.numel() * 2 + lse.numel() * 4
+    plan.close()
+
+    cpu_base = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        qc, kc, vc = hq, hk, hv
+        r = oracle_sample(w, qc, kc, vc, args.cpu_seconds)
+        cpu_base = {"value": r["flops"] / r["seconds"] / 1e12, "unit": "TFLOP/s", "cores": r["threads"],
+                    "kind": "oracle",
+                    "sample": f"{r['rows']} random output rows of {w.name} (fp64 oracle, {r['seconds']:.1f} s, "
+                              f"{cpu_model()})"}
+
+    if rank == 0:
+        peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+        peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+        traffic = None
+        tpath = os.path.join(ROOT, "profiles", "traffic.json")
+        if os.path.exists(tpath):
+            with open(tpath) as f:
+                tj = json.load(f)
+            entry = tj.get(w.name)
+            if entry and entry.get("kernel_rev") == kernel_revision():
+                traffic = entry.get("bytes_per_launch")
+        line = {
+            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": elapsed_max / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded N(0,1) bf16 q/k/v from a counter-based generator)",
+            "config": dict(w.describe(), parallelism=f"replicas{world}" if world > 1 else "single_gpu",
+                           l2="inputs larger than L2 (q+k+v+o of the workload exceed the 129 MB L2)"),
+            "tokens_per_s": value * 1e12 / (flops / w.total_q),
+            "pct_bf16_peak": value / peak,
+            "pct_bf16_peak_sustained": value / peak_sus,
+            "kernel_ms": kernel_ms,
+            "flops_per_step": flops,
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                         "frac": achieved / peak, "traffic": traffic,
+                         "peak_source": f"{peak_src} bf16_tflops (burst)"},
+            "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": e2e_steps},
+            "cpu_baseline": cpu_base,
+            "clocks": clocks,
+            "gpu_launches": args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def kernel_revision() -> str:
+    """Hash of the kernel sources: traffic counters are only valid for the kernel they were taken on."""
+    import hashlib
+    h = hashlib.sha1()
+    for f in ("opattn_kernel.cu", "ptx.cuh", "opattn_internal.h"):
+        with open(os.path.join(ROOT, "paper_2608_13499_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:12]
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="llama3_70b",
+                    help="tiny | llama3_8b | llama3_70b | bursty | chunked")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--reference-step-seconds", type=float, default=3.0)
+    args = ap.parse_args(argv)
+    from paper_2608_13499_gb300 import workloads as W
+    w = W.STANDARD[args.workload]()
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_ours(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,151 @@
+/*
+ * opattn.h -- C ABI of libopattn: causal grouped-query prefill attention over
+ * a ragged, packed batch of prompts, on one NVIDIA GB300 (sm_103a).
+ *
+ * The operation is the attention operator that OpScale (§2.1, "Compute
+ * Sensitivity") identifies as the prompt-length-sensitive, O(L^2 b) operator
+ * that sets time-to-first-token; it is exact softmax attention computed
+ * without materialising the L x L score matrix (§2.1, "Memory Sensitivity",
+ * FlashAttention).  Query heads are grouped over key/value heads
+ * (grouped-query attention, §5.6) and the causal mask is aligned to the
+ * bottom-right corner of each sequence so that a chunk of a prompt attends to
+ * its already-cached prefix (chunked prefill, §6).
+ *
+ * For sequence s with Lq = cu_seqlens_q[s+1] - cu_seqlens_q[s] queries and
+ * Lk = cu_seqlens_k[s+1] - cu_seqlens_k[s] keys, query row i (0-based within
+ * the sequence) sees key j iff j <= i + (Lk - Lq) and j < Lk.  With
+ * G = Hq / Hkv, query head h reads key/value head h / G.  For every query
+ * row i and head h:
+ *     x_j = scale * <q[i,h,:], k[j,h/G,:]>
+ *     O[i,h,:]  = sum_j softmax(x)_j * v[j,h/G,:]
+ *     LSE[i,h]  = ln sum_j exp(x_j)          (natural log, scaled logits)
+ * A row that sees no key gets O = 0 and LSE = -infinity.
+ *
+ * Layouts (all packed, contiguous, row-major):
+ *     q   bf16 [total_q, Hq,  d]     total_q = cu_seqlens_q[n_seq]
+ *     k,v bf16 [total_k, Hkv, d]     total_k = cu_seqlens_k[n_seq]
+ *     o   bf16 [total_q, Hq,  d]
+ *     lse fp32 [total_q, Hq]
+ * q, k, v, o and lse are device pointers; q, k, v and o must be 16-byte
+ * aligned and lse 4-byte aligned.  cu_seqlens_q / cu_seqlens_k are HOST
+ * arrays of n_seq + 1 int32 offsets, starting at 0 and non-decreasing.
+ * Sequences may be empty and may have Lq > Lk.
+ *
+ * Ownership: the caller owns every buffer and the stream.  The library keeps
+ * no pointer to caller memory after a call returns.
+ *
+ * Asynchrony: every call except opattn_prefill_checked and the plan
+ * create/destroy calls is asynchronous with respect to the host and ordered
+ * on `stream` (a cudaStream_t; NULL means the legacy default stream).
+ * Outputs are valid once the stream has reached the call.
+ *
+ * Errors: every function returns an opattn_status.  Argument errors are
+ * detected on the host before any device work and leave outputs untouched.
+ * The kernel bounds every wait; if one expires it stops early and records
+ * the error in a device status word, which opattn_prefill_checked reads back.
+ */
+#ifndef OPATTN_H
+#define OPATTN_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define OPATTN_API __attribute__((visibility("default")))
+#else
+#define OPATTN_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum opattn_status {
+    OPATTN_OK = 0,
+    OPATTN_ERR_INVALID_ARG = 1,  /* null pointer, bad count, non-monotone offsets, scale <= 0 */
+    OPATTN_ERR_UNSUPPORTED = 2,  /* d not in {64, 128}, or Hq / Hkv > 128 */
+    OPATTN_ERR_MISALIGNED = 3,   /* q/k/v/o not 16-byte or lse not 4-byte aligned */
+    OPATTN_ERR_CUDA = 4,         /* a CUDA runtime call or the launch failed */
+    OPATTN_ERR_TIMEOUT = 5,      /* a bounded device wait expired (checked entry point only) */
+    OPATTN_ERR_CAPACITY = 6      /* an output array given to opattn_schedule is too small */
+} opattn_status;
+
+/* Library version as major * 10000 + minor * 100 + patch. */
+OPATTN_API int32_t opattn_version(void);
+
+/* Static, NUL-terminated description of a status code. */
+OPATTN_API const char *opattn_status_string(int32_t status);
+
+/*
+ * One-shot prefill attention (the definition above).  Builds the
+ * longest-first work list on the host, copies it to stream-ordered device
+ * scratch (cudaMallocAsync / cudaFreeAsync on `stream`) and launches one
+ * persistent kernel over min(#SMs, #units) CTAs.  Returns OPATTN_OK with no
+ * device work when total_q == 0.  `scale` must be finite and > 0 (usually
+ * 1 / sqrt(d)).  Device-side wait timeouts are not reported here; use
+ * opattn_prefill_checked to observe them.
+ */
+OPATTN_API opattn_status opattn_prefill(const void *q, const void *k, const void *v, void *o, float *lse,
+                             const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                             int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
+                             void *stream);
+
+/*
+ * Diagnostic variant: the same computation, then it synchronizes `stream`
+ * and reads back the kernel's status word; returns OPATTN_ERR_TIMEOUT if a
+ * bounded wait expired.  `flags` must be 0 except in the library's own
+ * failure-path test, where OPATTN_FLAG_TEST_FORCE_TIMEOUT makes one kernel
+ * wait run out on purpose (after ~20 ms) so that the error path is
+ * exercised without hanging the GPU; outputs are then unspecified.
+ */
+#define OPATTN_FLAG_TEST_FORCE_TIMEOUT 1u
+OPATTN_API opattn_status opattn_prefill_checked(const void *q, const void *k, const void *v, void *o, float *lse,
+                                     const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                                     int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
+                                     void *stream, uint32_t flags);
+
+/*
+ * Reusable plan.  All layers of a model share the same cu_seqlens within a
+ * batch, so the work list can be built and uploaded once and then run per
+ * layer.  opattn_plan_create validates the geometry, builds the list for at
+ * most `max_ctas` CTAs (0 = one per SM of the current device), allocates
+ * device memory with cudaMalloc on the current device and copies the list
+ * synchronously.  opattn_plan_run launches the kernel only (no host work
+ * beyond tensor-map encoding, no allocation); it must run on the device the
+ * plan was created on.  opattn_plan_destroy frees the plan after
+ * synchronizing that device.  *plan is set to NULL on failure.
+ */
+typedef struct opattn_plan opattn_plan;
+OPATTN_API opattn_status opattn_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
+                                 const int32_t *cu_seqlens_k, int32_t n_seq, int32_t Hq,
+                                 int32_t Hkv, int32_t d, int32_t max_ctas);
+OPATTN_API opattn_status opattn_plan_run(const opattn_plan *plan, const void *q, const void *k, const void *v,
+                              void *o, float *lse, float scale, void *stream);
+OPATTN_API opattn_status opattn_plan_destroy(opattn_plan *plan);
+/* Number of work units and CTAs of a plan (either pointer may be NULL). */
+OPATTN_API opattn_status opattn_plan_info(const opattn_plan *plan, int64_t *n_units, int32_t *n_ctas);
+
+/*
+ * Host-only scheduler (no GPU needed), exposed for testing and capacity
+ * planning.  A work unit is (sequence, kv head, block of 2 * (128 / G)
+ * query tokens).  Its cost is the number of 128-key tiles it visits after
+ * whole tiles above the causal diagonal are skipped, plus one.  Units are
+ * sorted by cost, longest first, and each is given to the CTA with the least
+ * assigned cost so far (Graham's longest-processing-time rule).
+ * Writes `units` as 8 int32 per unit:
+ *     {first packed query row, tokens in unit, first packed key row of the
+ *      sequence, Lk, last visible key of the unit's first token, kv head,
+ *      key tiles visited, sequence index}
+ * grouped by CTA, and cta_offsets[0..n_ctas] (unit index ranges).  n_ctas
+ * used = min(n_ctas, #units), returned in *n_ctas_used.  Fails with
+ * OPATTN_ERR_CAPACITY (and *n_units_out set) if unit_capacity is too small.
+ */
+OPATTN_API opattn_status opattn_schedule(const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                              int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, int32_t n_ctas,
+                              int32_t *units, int64_t unit_capacity, int32_t *cta_offsets,
+                              int64_t *n_units_out, int32_t *n_ctas_used);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OPATTN_H */

@@ -1,0 +1,436 @@
+// opattn_api.cpp -- host runtime of libopattn: argument validation, the
+// longest-first ragged work-list scheduler, pinned staging for the work
+// list, reusable plans and the C-ABI entry points declared in opattn.h.
+#include "opattn.h"
+
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <functional>
+#include <mutex>
+#include <queue>
+#include <utility>
+#include <vector>
+
+#include "opattn_internal.h"
+
+namespace opattn {
+namespace {
+
+constexpr int32_t kVersion = 10000;  // 1.0.0
+
+struct Geometry {
+    int32_t n_seq, Hq, Hkv, d, G, TPB;
+    int64_t total_q, total_k;
+};
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Checks that do not touch tensor pointers.
+opattn_status check_geometry(const int32_t* cu_q, const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv,
+                             int32_t d, Geometry* g) {
+    if (n_seq < 0 || Hq <= 0 || Hkv <= 0) return OPATTN_ERR_INVALID_ARG;
+    if (n_seq > 0 && (!cu_q || !cu_k)) return OPATTN_ERR_INVALID_ARG;
+    if (Hq % Hkv != 0) return OPATTN_ERR_INVALID_ARG;
+    if (d != 64 && d != 128) return OPATTN_ERR_UNSUPPORTED;
+    const int32_t G = Hq / Hkv;
+    if (G > kRowsPerTile) return OPATTN_ERR_UNSUPPORTED;
+    if (n_seq > 0) {
+        if (cu_q[0] != 0 || cu_k[0] != 0) return OPATTN_ERR_INVALID_ARG;
+        for (int32_t s = 0; s < n_seq; ++s)
+            if (cu_q[s + 1] < cu_q[s] || cu_k[s + 1] < cu_k[s]) return OPATTN_ERR_INVALID_ARG;
+    }
+    g->n_seq = n_seq;
+    g->Hq = Hq;
+    g->Hkv = Hkv;
+    g->d = d;
+    g->G = G;
+    g->TPB = tokens_per_tile(G);
+    g->total_q = n_seq > 0 ? cu_q[n_seq] : 0;
+    g->total_k = n_seq > 0 ? cu_k[n_seq] : 0;
+    // Packed row indices (token * heads + head) must fit the 32-bit unit
+    // fields and the 32-bit TMA coordinates.
+    if (g->total_q * static_cast<int64_t>(Hq) >= (int64_t{1} << 31)) return OPATTN_ERR_UNSUPPORTED;
+    if (g->total_k * static_cast<int64_t>(Hkv) >= (int64_t{1} << 31)) return OPATTN_ERR_UNSUPPORTED;
+    return OPATTN_OK;
+}
+
+opattn_status check_tensors(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                            float scale, const Geometry& g) {
+    if (!(std::isfinite(scale) && scale > 0.f)) return OPATTN_ERR_INVALID_ARG;
+    if (!q || !o || !lse) return OPATTN_ERR_INVALID_ARG;
+    if (g.total_k > 0 && (!k || !v)) return OPATTN_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(o, 16) || !aligned(lse, 4)) return OPATTN_ERR_MISALIGNED;
+    if (g.total_k > 0 && (!aligned(k, 16) || !aligned(v, 16))) return OPATTN_ERR_MISALIGNED;
+    return OPATTN_OK;
+}
+
+// ------------------------------------------------------------- scheduler
+
+struct Schedule {
+    std::vector<UnitRec> units;    // grouped by CTA, longest first within a CTA
+    std::vector<int32_t> cta_off;  // n_cta + 1
+    int32_t n_cta = 0;
+};
+
+// Units are (sequence, kv head, block of 2 * TPB query tokens).  Cost is the
+// number of key tiles the block visits after whole tiles above the causal
+// diagonal are skipped, plus one for the Q load and the epilogue.  Units are
+// bucket-sorted by cost, longest first, and each goes to the CTA with the
+// least cost so far (longest-processing-time greedy; makespan within 4/3 of
+// optimal).
+void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out) {
+    const int32_t tpu = 2 * g.TPB;
+    std::vector<UnitRec> all;
+    int32_t max_cost = 0;
+    for (int32_t s = 0; s < g.n_seq; ++s) {
+        const int32_t Lq = cu_q[s + 1] - cu_q[s];
+        const int32_t Lk = cu_k[s + 1] - cu_k[s];
+        const int32_t delta = Lk - Lq;
+        for (int32_t t0 = 0; t0 < Lq; t0 += tpu) {
+            const int32_t n_tok = std::min(tpu, Lq - t0);
+            const int32_t qlim0 = t0 + delta;
+            const int32_t last_key = std::min(qlim0 + n_tok - 1, Lk - 1);
+            const int32_t n_tiles = last_key < 0 ? 0 : last_key / kBlockN + 1;
+            max_cost = std::max(max_cost, n_tiles + 1);
+            for (int32_t h = 0; h < g.Hkv; ++h) {
+                UnitRec u;
+                u.q_tok0 = cu_q[s] + t0;
+                u.n_tok = n_tok;
+                u.k_row0 = cu_k[s];
+                u.Lk = Lk;
+                u.qlim0 = qlim0;
+                u.kvh = h;
+                u.n_tiles = n_tiles;
+                u.seq = s;
+                all.push_back(u);
+            }
+        }
+    }
+    const int64_t n = static_cast<int64_t>(all.size());
+    out->units.clear();
+    out->cta_off.clear();
+    out->n_cta = 0;
+    if (n == 0) return;
+    const int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(std::max<int32_t>(max_ctas, 1), n));
+
+    // counting sort by cost, descending (stable: sequence order within a cost)
+    std::vector<int64_t> count(static_cast<size_t>(max_cost) + 2, 0);
+    for (const UnitRec& u : all) ++count[static_cast<size_t>(max_cost - (u.n_tiles + 1))];
+    int64_t acc = 0;
+    for (auto& c : count) {
+        const int64_t t = c;
+        c = acc;
+        acc += t;
+    }
+    std::vector<int64_t> order(static_cast<size_t>(n));
+    for (int64_t i = 0; i < n; ++i) order[static_cast<size_t>(count[static_cast<size_t>(max_cost - (all[i].n_tiles + 1))]++)] = i;
+
+    // greedy: next unit to the least-loaded CTA (ties: lower CTA index)
+    using Slot = std::pair<int64_t, int32_t>;
+    std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> heap;
+    for (int32_t c = 0; c < n_cta; ++c) heap.push({0, c});
+    std::vector<int32_t> owner(static_cast<size_t>(n));
+    std::vector<int32_t> per_cta(static_cast<size_t>(n_cta), 0);
+    for (int64_t i = 0; i < n; ++i) {
+        Slot sl = heap.top();
+        heap.pop();
+        const UnitRec& u = all[static_cast<size_t>(order[static_cast<size_t>(i)])];
+        owner[static_cast<size_t>(i)] = sl.second;
+        ++per_cta[static_cast<size_t>(sl.second)];
+        sl.first += u.n_tiles + 1;
+        heap.push(sl);
+    }
+    out->cta_off.assign(static_cast<size_t>(n_cta) + 1, 0);
+    for (int32_t c = 0; c < n_cta; ++c) out->cta_off[static_cast<size_t>(c) + 1] = out->cta_off[static_cast<size_t>(c)] + per_cta[static_cast<size_t>(c)];
+    std::vector<int32_t> fill(out->cta_off.begin(), out->cta_off.end() - 1);
+    out->units.resize(static_cast<size_t>(n));
+    for (int64_t i = 0; i < n; ++i) {
+        const int32_t c = owner[static_cast<size_t>(i)];
+        out->units[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = all[static_cast<size_t>(order[static_cast<size_t>(i)])];
+    }
+    out->n_cta = n_cta;
+}
+
+// Device work area: [cta_off (n_cta + 1) | pad to 32 B | units | status].
+struct WorkLayout {
+    size_t off_units, off_status, bytes, upload_bytes;
+};
+WorkLayout work_layout(const Schedule& s) {
+    WorkLayout w;
+    const size_t off_bytes = (s.cta_off.size() * sizeof(int32_t) + 31) / 32 * 32;
+    w.off_units = off_bytes;
+    w.off_status = off_bytes + s.units.size() * sizeof(UnitRec);
+    w.upload_bytes = w.off_status;
+    w.bytes = w.off_status + 32;
+    return w;
+}
+void pack_upload(const Schedule& s, const WorkLayout& w, uint8_t* dst) {
+    std::memset(dst, 0, w.upload_bytes);
+    std::memcpy(dst, s.cta_off.data(), s.cta_off.size() * sizeof(int32_t));
+    std::memcpy(dst + w.off_units, s.units.data(), s.units.size() * sizeof(UnitRec));
+}
+
+// ---------------------------------------------------- pinned staging pool
+// The work list goes to the device with an asynchronous copy from pinned
+// memory; a staging buffer is reused only after the event recorded behind
+// its copy has completed, so no call ever blocks on the GPU.
+struct Staging {
+    void* host = nullptr;
+    size_t cap = 0;
+    cudaEvent_t done = nullptr;
+    bool busy = false;
+};
+std::mutex g_stage_mu;
+std::vector<Staging*> g_stage_pool;
+
+Staging* staging_acquire(size_t bytes) {
+    std::lock_guard<std::mutex> lk(g_stage_mu);
+    for (Staging* s : g_stage_pool) {
+        if (s->busy || s->cap < bytes) continue;
+        if (cudaEventQuery(s->done) != cudaSuccess) {
+            (void)cudaGetLastError();  // cudaErrorNotReady is not an error here
+            continue;
+        }
+        s->busy = true;
+        return s;
+    }
+    Staging* s = new Staging;
+    size_t cap = 4096;
+    while (cap < bytes) cap *= 2;
+    if (cudaHostAlloc(&s->host, cap, cudaHostAllocPortable) != cudaSuccess) {
+        delete s;
+        return nullptr;
+    }
+    if (cudaEventCreateWithFlags(&s->done, cudaEventDisableTiming) != cudaSuccess) {
+        cudaFreeHost(s->host);
+        delete s;
+        return nullptr;
+    }
+    s->cap = cap;
+    s->busy = true;
+    g_stage_pool.push_back(s);
+    return s;
+}
+void staging_release(Staging* s, cudaStream_t stream) {
+    std::lock_guard<std::mutex> lk(g_stage_mu);
+    cudaEventRecord(s->done, stream);
+    s->busy = false;
+}
+
+int device_sm_count() {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    return sms;
+}
+
+LaunchArgs make_args(const void* q, const void* k, const void* v, void* o, float* lse, const Geometry& g,
+                     float scale, const uint8_t* work, const WorkLayout& w, int32_t n_cta, uint32_t flags) {
+    LaunchArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.o = o;
+    a.lse = lse;
+    a.total_q = g.total_q;
+    a.total_k = g.total_k;
+    a.Hq = g.Hq;
+    a.Hkv = g.Hkv;
+    a.d = g.d;
+    a.scale = scale;
+    a.units = reinterpret_cast<const UnitRec*>(work + w.off_units);
+    a.cta_off = reinterpret_cast<const int32_t*>(work);
+    a.n_cta = n_cta;
+    a.status = reinterpret_cast<int32_t*>(const_cast<uint8_t*>(work) + w.off_status);
+    a.flags = flags;
+    return a;
+}
+
+// One-shot path shared by opattn_prefill and opattn_prefill_checked.
+opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
+                           const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
+                           cudaStream_t stream, uint32_t flags, bool checked) {
+    Geometry g;
+    opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    if (g.total_q == 0) return OPATTN_OK;
+    st = check_tensors(q, k, v, o, lse, scale, g);
+    if (st != OPATTN_OK) return st;
+    const int sms = device_sm_count();
+    if (sms <= 0) return OPATTN_ERR_CUDA;
+
+    Schedule sch;
+    build_schedule(cu_q, cu_k, g, sms, &sch);
+    const WorkLayout w = work_layout(sch);
+    Staging* stg = staging_acquire(w.upload_bytes);
+    if (!stg) return OPATTN_ERR_CUDA;
+    pack_upload(sch, w, static_cast<uint8_t*>(stg->host));
+
+    void* work = nullptr;
+    if (cudaMallocAsync(&work, w.bytes, stream) != cudaSuccess) {
+        staging_release(stg, stream);
+        return OPATTN_ERR_CUDA;
+    }
+    bool ok = cudaMemcpyAsync(work, stg->host, w.upload_bytes, cudaMemcpyHostToDevice, stream) == cudaSuccess;
+    ok = ok && cudaMemsetAsync(static_cast<uint8_t*>(work) + w.off_status, 0, sizeof(int32_t), stream) == cudaSuccess;
+    staging_release(stg, stream);
+    int32_t dev_status = 0;
+    if (ok) {
+        const LaunchArgs a = make_args(q, k, v, o, lse, g, scale, static_cast<uint8_t*>(work), w, sch.n_cta, flags);
+        ok = launch_prefill(a, stream) == 0;
+    }
+    if (ok && checked) {
+        ok = cudaMemcpyAsync(&dev_status, static_cast<uint8_t*>(work) + w.off_status, sizeof(int32_t),
+                             cudaMemcpyDeviceToHost, stream) == cudaSuccess;
+        ok = ok && cudaStreamSynchronize(stream) == cudaSuccess;
+    }
+    cudaFreeAsync(work, stream);
+    if (!ok) return OPATTN_ERR_CUDA;
+    if (checked && dev_status != kDevOk) return OPATTN_ERR_TIMEOUT;
+    return OPATTN_OK;
+}
+
+}  // namespace
+}  // namespace opattn
+
+using namespace opattn;
+
+struct opattn_plan {
+    Geometry g;
+    Schedule sch;
+    WorkLayout w;
+    int device = 0;
+    void* work = nullptr;
+};
+
+extern "C" {
+
+int32_t opattn_version(void) { return kVersion; }
+
+const char* opattn_status_string(int32_t status) {
+    switch (status) {
+        case OPATTN_OK: return "ok";
+        case OPATTN_ERR_INVALID_ARG: return "invalid argument";
+        case OPATTN_ERR_UNSUPPORTED: return "unsupported configuration (head dim must be 64 or 128, Hq/Hkv <= 128)";
+        case OPATTN_ERR_MISALIGNED: return "misaligned pointer (q/k/v/o need 16 bytes, lse 4 bytes)";
+        case OPATTN_ERR_CUDA: return "CUDA runtime error";
+        case OPATTN_ERR_TIMEOUT: return "device wait timed out";
+        case OPATTN_ERR_CAPACITY: return "output array too small";
+        default: return "unknown status";
+    }
+}
+
+opattn_status opattn_prefill(const void* q, const void* k, const void* v, void* o, float* lse,
+                             const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq, int32_t Hq,
+                             int32_t Hkv, int32_t d, float scale, void* stream) {
+    return prefill_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
+                        static_cast<cudaStream_t>(stream), 0u, false);
+}
+
+opattn_status opattn_prefill_checked(const void* q, const void* k, const void* v, void* o, float* lse,
+                                     const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
+                                     int32_t Hq, int32_t Hkv, int32_t d, float scale, void* stream,
+                                     uint32_t flags) {
+    if (flags & ~OPATTN_FLAG_TEST_FORCE_TIMEOUT) return OPATTN_ERR_INVALID_ARG;
+    const uint32_t kflags = (flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u;
+    return prefill_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
+                        static_cast<cudaStream_t>(stream), kflags, true);
+}
+
+opattn_status opattn_plan_create(opattn_plan** plan, const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k,
+                                 int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, int32_t max_ctas) {
+    if (!plan) return OPATTN_ERR_INVALID_ARG;
+    *plan = nullptr;
+    if (max_ctas < 0) return OPATTN_ERR_INVALID_ARG;
+    Geometry g;
+    opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    opattn_plan* p = new opattn_plan;
+    p->g = g;
+    if (cudaGetDevice(&p->device) != cudaSuccess) {
+        delete p;
+        return OPATTN_ERR_CUDA;
+    }
+    if (g.total_q > 0) {
+        const int sms = device_sm_count();
+        if (sms <= 0) {
+            delete p;
+            return OPATTN_ERR_CUDA;
+        }
+        const int32_t cap = max_ctas > 0 ? std::min(max_ctas, sms) : sms;
+        build_schedule(cu_seqlens_q, cu_seqlens_k, g, cap, &p->sch);
+        p->w = work_layout(p->sch);
+        std::vector<uint8_t> host(p->w.bytes, 0);
+        pack_upload(p->sch, p->w, host.data());
+        if (cudaMalloc(&p->work, p->w.bytes) != cudaSuccess) {
+            delete p;
+            return OPATTN_ERR_CUDA;
+        }
+        if (cudaMemcpy(p->work, host.data(), p->w.bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+            cudaFree(p->work);
+            delete p;
+            return OPATTN_ERR_CUDA;
+        }
+    }
+    *plan = p;
+    return OPATTN_OK;
+}
+
+opattn_status opattn_plan_run(const opattn_plan* plan, const void* q, const void* k, const void* v, void* o,
+                              float* lse, float scale, void* stream) {
+    if (!plan) return OPATTN_ERR_INVALID_ARG;
+    if (plan->g.total_q == 0) return OPATTN_OK;
+    opattn_status st = check_tensors(q, k, v, o, lse, scale, plan->g);
+    if (st != OPATTN_OK) return st;
+    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, static_cast<uint8_t*>(plan->work), plan->w,
+                                   plan->sch.n_cta, 0u);
+    return launch_prefill(a, static_cast<cudaStream_t>(stream)) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+}
+
+opattn_status opattn_plan_destroy(opattn_plan* plan) {
+    if (!plan) return OPATTN_OK;
+    opattn_status st = OPATTN_OK;
+    if (plan->work) {
+        int prev = 0;
+        cudaGetDevice(&prev);
+        cudaSetDevice(plan->device);
+        if (cudaDeviceSynchronize() != cudaSuccess) st = OPATTN_ERR_CUDA;
+        if (cudaFree(plan->work) != cudaSuccess) st = OPATTN_ERR_CUDA;
+        cudaSetDevice(prev);
+    }
+    delete plan;
+    return st;
+}
+
+opattn_status opattn_plan_info(const opattn_plan* plan, int64_t* n_units, int32_t* n_ctas) {
+    if (!plan) return OPATTN_ERR_INVALID_ARG;
+    if (n_units) *n_units = static_cast<int64_t>(plan->sch.units.size());
+    if (n_ctas) *n_ctas = plan->sch.n_cta;
+    return OPATTN_OK;
+}
+
+opattn_status opattn_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq, int32_t Hq,
+                              int32_t Hkv, int32_t d, int32_t n_ctas, int32_t* units, int64_t unit_capacity,
+                              int32_t* cta_offsets, int64_t* n_units_out, int32_t* n_ctas_used) {
+    if (n_ctas <= 0 || !n_units_out || !n_ctas_used) return OPATTN_ERR_INVALID_ARG;
+    Geometry g;
+    opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    Schedule sch;
+    build_schedule(cu_seqlens_q, cu_seqlens_k, g, n_ctas, &sch);
+    *n_units_out = static_cast<int64_t>(sch.units.size());
+    *n_ctas_used = sch.n_cta;
+    if (static_cast<int64_t>(sch.units.size()) > unit_capacity) return OPATTN_ERR_CAPACITY;
+    if (!sch.units.empty() && (!units || !cta_offsets)) return OPATTN_ERR_INVALID_ARG;
+    if (!sch.units.empty()) {
+        std::memcpy(units, sch.units.data(), sch.units.size() * sizeof(UnitRec));
+        std::memcpy(cta_offsets, sch.cta_off.data(), sch.cta_off.size() * sizeof(int32_t));
+    }
+    return OPATTN_OK;
+}
+
+}  // extern "C"

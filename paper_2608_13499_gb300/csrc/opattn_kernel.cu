@@ -1,0 +1,585 @@
+// opattn_kernel.cu -- persistent sm_103a kernel for ragged causal GQA prefill
+// attention (tcgen05 MMAs with TMEM accumulators, TMA + mbarrier K/V ring).
+//
+// What it computes is exact softmax attention (OpScale §2.1: the attention
+// operator is O(L^2 b) in the prompt length and is computed FlashAttention
+// style, without materialising the L x L score matrix), with query heads
+// grouped over kv heads (§5.6) and a bottom-right-aligned causal mask
+// (chunked prefill, §6).  Softmax is evaluated online over 128-key tiles
+// with base-2 exponentials; the result equals the two-pass definition up to
+// rounding.
+//
+// CTA layout (384 threads, one CTA per SM, persistent over its unit list):
+//   warp 0        TMA producer: Q tiles of the unit, then K_j, V_j into a ring
+//   warp 1        TMEM owner + single-thread MMA issuer
+//   warps 2-3     idle
+//   warps 4-7     softmax / correction / epilogue of M-tile 0 (one row per thread)
+//   warps 8-11    the same for M-tile 1
+// TMEM (512 columns): S0 | S1 (128 fp32 columns each; P is written back into
+// the first 64 columns as packed bf16) | O0 | O1 (d columns each).
+//
+// MMA order per key tile j (after the prologue S0(0), S1(0)):
+//   PV0(j), S0(j+1) -> commit S-ready[0] (or O-ready[0] after the last tile)
+//   PV1(j), S1(j+1) -> commit S-ready[1] (or O-ready[1])
+// so the tensor pipe works on one M-tile while the other M-tile's softmax
+// runs.  tcgen05 MMAs from one thread execute in issue order, so S_i(j+1),
+// which overwrites P_i(j), never runs before PV_i(j) has read it, and once
+// S_i(j+1) has completed so has PV_i(j): the softmax thread may rescale O_i
+// right after it sees S-ready.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "opattn_internal.h"
+#include "ptx.cuh"
+
+namespace opattn {
+namespace {
+
+constexpr int kThreads = 384;
+constexpr int kWarpProducer = 0;
+constexpr int kWarpMma = 1;
+constexpr int kWarpSoftmax = 4;  // first softmax warp; warps 4..7 -> M-tile 0, 8..11 -> M-tile 1
+
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: no legitimate wait comes close
+constexpr uint64_t kForcedLimitNs = 20000000ull;  // 20 ms: the forced-timeout test
+constexpr uint64_t kDrainLimitNs = 200000000ull;  // in-flight copies / MMAs after an abort
+// Rescale O only when a row's running maximum grows by more than 2^8: the
+// final division by l uses the same stale maximum, so the result is exact;
+// probabilities stay below 2^8, far inside bf16 and fp32 range.
+constexpr float kRescaleThreshold = 8.0f;
+constexpr float kLn2 = 0.693147180559945309f;
+constexpr float kLog2e = 1.442695040888963407f;
+
+template <int D>
+struct Cfg {
+    static_assert(D == 64 || D == 128, "head dim");
+    static constexpr int kDBlocks = D / 64;                        // 128-byte swizzle column blocks
+    static constexpr int kQTileBytes = kRowsPerTile * D * 2;       // one M-tile of Q
+    static constexpr int kSlotBytes = kBlockN * D * 2;             // one K or V tile
+    static constexpr int kSlots = D == 128 ? 4 : 8;                // ring depth (K and V alternate)
+    static constexpr int kQOff = 0;
+    static constexpr int kRingOff = 2 * kQTileBytes;
+    static constexpr int kBarOff = kRingOff + kSlots * kSlotBytes;
+    static constexpr int kBarFull = 0;
+    static constexpr int kBarEmpty = kSlots;
+    static constexpr int kBarQFull = 2 * kSlots;       // + M-tile
+    static constexpr int kBarQEmpty = 2 * kSlots + 2;  // + M-tile
+    static constexpr int kBarS = 2 * kSlots + 4;       // S ready (+ M-tile)
+    static constexpr int kBarO = 2 * kSlots + 6;       // final O ready (+ M-tile)
+    static constexpr int kBarP = 2 * kSlots + 8;       // P written, O corrected (+ M-tile)
+    static constexpr int kBarDrain = 2 * kSlots + 10;
+    static constexpr int kBarNever = 2 * kSlots + 11;
+    static constexpr int kNumBars = 2 * kSlots + 12;
+    static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // TMEM base address, abort flag
+    static constexpr int kSmemBytes = kMiscOff + 16 + 1024;  // + slack for 1024-byte alignment
+    static constexpr uint32_t kTmemCols = 512;
+    static constexpr uint32_t kColS = 0;    // + 128 * M-tile
+    static constexpr uint32_t kColO = 256;  // + D * M-tile
+    static constexpr uint32_t kIdescS = ptx::idesc_bf16_f32(kRowsPerTile, kBlockN, false);
+    static constexpr uint32_t kIdescPV = ptx::idesc_bf16_f32(kRowsPerTile, D, true);
+    static constexpr uint32_t kQTxBytesPerRow = D * 2;
+};
+
+struct KParams {
+    const UnitRec* units;
+    const int32_t* cta_off;
+    uint16_t* o;
+    float* lse;
+    int32_t Hq, G, TPB;
+    float scale_log2;  // softmax scale * log2(e)
+    int32_t* status;
+    uint32_t flags;
+};
+
+// Wait for the phase of parity `parity` of `bar`.  Gives up when another
+// thread of the CTA has aborted, or after `limit_ns`, in which case it
+// raises the CTA abort flag and records a timeout in the status word.
+__device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, volatile int32_t* abort_flag,
+                                             int32_t* status, uint64_t limit_ns) {
+    if (ptx::mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = ptx::globaltimer_ns();
+    for (;;) {
+        if (ptx::mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (ptx::globaltimer_ns() - t0 > limit_ns) {
+            *abort_flag = 1;
+            atomicCAS(status, kDevOk, kDevTimeout);
+            return false;
+        }
+    }
+}
+
+// Wait used while shutting down after an abort: ignores the abort flag and
+// returns silently after `limit_ns`.
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+    const uint64_t t0 = ptx::globaltimer_ns();
+    while (!ptx::mbar_try_wait(bar, parity)) {
+        if (ptx::globaltimer_ns() - t0 > limit_ns) return;
+    }
+}
+
+template <int D>
+__device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUtensorMap* tmK,
+                                             const CUtensorMap* tmV, const KParams& p, int ubeg, int uend,
+                                             uint32_t sQ, uint32_t sRing, uint32_t sBar,
+                                             volatile int32_t* abort_flag) {
+    using C = Cfg<D>;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    const uint32_t q_tx = static_cast<uint32_t>(p.G * p.TPB) * C::kQTxBytesPerRow;
+    uint32_t slot = 0, ring_par = 0;
+    uint32_t q_issued[2] = {0u, 0u};
+    uint32_t ring_issued = 0;
+    bool aborted = false;
+    for (int ui = ubeg; ui < uend && !aborted; ++ui) {
+        const UnitRec u = p.units[ui];
+        if (u.n_tiles <= 0) continue;
+        for (int i = 0; i < 2; ++i) {
+            if (!bounded_wait(bar(C::kBarQEmpty + i), (q_issued[i] & 1u) ^ 1u, abort_flag, p.status,
+                              kWaitLimitNs)) {
+                aborted = true;
+                break;
+            }
+            ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + i), q_tx);
+#pragma unroll
+            for (int b = 0; b < C::kDBlocks; ++b)
+                ptx::tma_load_3d(sQ + i * C::kQTileBytes + b * (kRowsPerTile * 128), tmQ,
+                                 bar(C::kBarQFull + i), b * 64, u.kvh * p.G, u.q_tok0 + i * p.TPB);
+            ++q_issued[i];
+        }
+        for (int j = 0; j < u.n_tiles && !aborted; ++j) {
+            for (int kv = 0; kv < 2; ++kv) {
+                if (!bounded_wait(bar(C::kBarEmpty + slot), ring_par ^ 1u, abort_flag, p.status,
+                                  kWaitLimitNs)) {
+                    aborted = true;
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(bar(C::kBarFull + slot), C::kSlotBytes);
+#pragma unroll
+                for (int b = 0; b < C::kDBlocks; ++b)
+                    ptx::tma_load_3d(sRing + slot * C::kSlotBytes + b * (kBlockN * 128), kv ? tmV : tmK,
+                                     bar(C::kBarFull + slot), b * 64, u.kvh, u.k_row0 + j * kBlockN);
+                ++ring_issued;
+                if (++slot == C::kSlots) {
+                    slot = 0;
+                    ring_par ^= 1u;
+                }
+            }
+        }
+    }
+    if (aborted) {
+        // Let every copy still in flight land before the CTA exits: at most
+        // one outstanding load per ring slot and per Q buffer (the latest).
+        for (uint32_t s = 0; s < static_cast<uint32_t>(C::kSlots); ++s) {
+            if (ring_issued > s) {
+                const uint32_t uses = (ring_issued - s + C::kSlots - 1) / C::kSlots;
+                drain_wait(bar(C::kBarFull + s), (uses - 1u) & 1u, kDrainLimitNs);
+            }
+        }
+        for (int i = 0; i < 2; ++i)
+            if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
+    }
+}
+
+template <int D>
+__device__ __forceinline__ void issue_s(uint32_t tmem, int mt, uint32_t sQ, uint32_t sK) {
+    using C = Cfg<D>;
+    const uint32_t d_tmem = tmem + C::kColS + 128u * mt;
+    const uint32_t qbase = sQ + mt * C::kQTileBytes;
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+        const uint32_t qoff = (ks >> 2) * (kRowsPerTile * 128) + (ks & 3) * 32;
+        const uint32_t koff = (ks >> 2) * (kBlockN * 128) + (ks & 3) * 32;
+        ptx::mma_ss(d_tmem, ptx::sdesc_sw128(qbase + qoff, 16, 1024), ptx::sdesc_sw128(sK + koff, 16, 1024),
+                    C::kIdescS, ks > 0 ? 1u : 0u);
+    }
+}
+
+template <int D>
+__device__ __forceinline__ void issue_pv(uint32_t tmem, int mt, uint32_t sV, bool accumulate) {
+    using C = Cfg<D>;
+    const uint32_t d_tmem = tmem + C::kColO + static_cast<uint32_t>(D) * mt;
+    const uint32_t a_tmem = tmem + C::kColS + 128u * mt;
+#pragma unroll
+    for (int ks = 0; ks < kBlockN / 16; ++ks) {
+        // V tile is [keys][d] (MN-major for this product): 16 keys per step,
+        // 64-column blocks kBlockN * 128 bytes apart, 8-key groups 1024 apart.
+        ptx::mma_ts(d_tmem, a_tmem + ks * 8, ptx::sdesc_sw128(sV + ks * (16 * 128), kBlockN * 128, 1024),
+                    C::kIdescPV, (accumulate || ks > 0) ? 1u : 0u);
+    }
+}
+
+template <int D>
+__device__ __forceinline__ void run_mma(const KParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sQ,
+                                        uint32_t sRing, uint32_t sBar, volatile int32_t* abort_flag) {
+    using C = Cfg<D>;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    auto slot_addr = [&](uint32_t s) { return sRing + s * C::kSlotBytes; };
+    uint32_t slot = 0, ring_par = 0, q_uses = 0;
+    uint32_t p_par[2] = {0u, 0u};
+    bool ok = true;
+    if (p.flags & kFlagForceTimeout) ok = bounded_wait(bar(C::kBarNever), 0u, abort_flag, p.status, kForcedLimitNs);
+
+    for (int ui = ubeg; ui < uend && ok; ++ui) {
+        const UnitRec u = p.units[ui];
+        const int nT = u.n_tiles;
+        if (nT <= 0) continue;
+        // prologue: S0(0), S1(0)
+        if (!(ok = bounded_wait(bar(C::kBarQFull + 0), q_uses & 1u, abort_flag, p.status, kWaitLimitNs))) break;
+        uint32_t kslot = slot;
+        if (!(ok = bounded_wait(bar(C::kBarFull + kslot), ring_par, abort_flag, p.status, kWaitLimitNs))) break;
+        if (++slot == C::kSlots) { slot = 0; ring_par ^= 1u; }
+        ptx::tc_fence_after();
+        issue_s<D>(tmem, 0, sQ, slot_addr(kslot));
+        ptx::tc_commit(bar(C::kBarS + 0));
+        if (nT == 1) ptx::tc_commit(bar(C::kBarQEmpty + 0));
+        if (!(ok = bounded_wait(bar(C::kBarQFull + 1), q_uses & 1u, abort_flag, p.status, kWaitLimitNs))) break;
+        ptx::tc_fence_after();
+        issue_s<D>(tmem, 1, sQ, slot_addr(kslot));
+        ptx::tc_commit(bar(C::kBarS + 1));
+        if (nT == 1) ptx::tc_commit(bar(C::kBarQEmpty + 1));
+        ptx::tc_commit(bar(C::kBarEmpty + kslot));
+        ++q_uses;
+
+        for (int j = 0; j < nT; ++j) {
+            const uint32_t vslot = slot;
+            if (!(ok = bounded_wait(bar(C::kBarFull + vslot), ring_par, abort_flag, p.status, kWaitLimitNs))) break;
+            if (++slot == C::kSlots) { slot = 0; ring_par ^= 1u; }
+            const bool more = j + 1 < nT;
+            // M-tile 0
+            if (!(ok = bounded_wait(bar(C::kBarP + 0), p_par[0], abort_flag, p.status, kWaitLimitNs))) break;
+            p_par[0] ^= 1u;
+            ptx::tc_fence_after();
+            issue_pv<D>(tmem, 0, slot_addr(vslot), j > 0);
+            if (more) {
+                kslot = slot;
+                if (!(ok = bounded_wait(bar(C::kBarFull + kslot), ring_par, abort_flag, p.status, kWaitLimitNs)))
+                    break;
+                if (++slot == C::kSlots) { slot = 0; ring_par ^= 1u; }
+                issue_s<D>(tmem, 0, sQ, slot_addr(kslot));
+                if (j + 2 == nT) ptx::tc_commit(bar(C::kBarQEmpty + 0));
+                ptx::tc_commit(bar(C::kBarS + 0));
+            } else {
+                ptx::tc_commit(bar(C::kBarO + 0));
+            }
+            // M-tile 1
+            if (!(ok = bounded_wait(bar(C::kBarP + 1), p_par[1], abort_flag, p.status, kWaitLimitNs))) break;
+            p_par[1] ^= 1u;
+            ptx::tc_fence_after();
+            issue_pv<D>(tmem, 1, slot_addr(vslot), j > 0);
+            if (more) {
+                issue_s<D>(tmem, 1, sQ, slot_addr(kslot));
+                if (j + 2 == nT) ptx::tc_commit(bar(C::kBarQEmpty + 1));
+                ptx::tc_commit(bar(C::kBarS + 1));
+                ptx::tc_commit(bar(C::kBarEmpty + kslot));
+            } else {
+                ptx::tc_commit(bar(C::kBarO + 1));
+            }
+            ptx::tc_commit(bar(C::kBarEmpty + vslot));
+        }
+    }
+    // Every MMA this thread issued must finish before TMEM is released.
+    ptx::tc_commit(bar(C::kBarDrain));
+    drain_wait(bar(C::kBarDrain), 0u, kDrainLimitNs);
+}
+
+template <int D>
+__device__ __forceinline__ void store_zero_row(const KParams& p, int64_t row_idx) {
+    uint4* dst = reinterpret_cast<uint4*>(p.o + row_idx * D);
+#pragma unroll
+    for (int i = 0; i < D / 8; ++i) dst[i] = make_uint4(0u, 0u, 0u, 0u);
+    p.lse[row_idx] = -INFINITY;
+}
+
+template <int D>
+__device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sBar,
+                                            int warp, int lane, volatile int32_t* abort_flag) {
+    using C = Cfg<D>;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    const int mt = (warp - kWarpSoftmax) >> 2;  // M-tile
+    const int quarter = warp & 3;               // TMEM lane quarter this warp may access
+    const int r = quarter * 32 + lane;          // accumulator row
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t tS = tmem + lane_off + C::kColS + 128u * mt;
+    const uint32_t tO = tmem + lane_off + C::kColO + static_cast<uint32_t>(D) * mt;
+    const int G = p.G, TPB = p.TPB;
+    const int tok_in_tile = r / G;
+    const int head_in_group = r - tok_in_tile * G;
+    const bool in_tile = r < G * TPB;
+    const float cl = p.scale_log2;
+    uint32_t s_par = 0, o_par = 0;
+
+    for (int ui = ubeg; ui < uend; ++ui) {
+        const UnitRec u = p.units[ui];
+        const int tok = mt * TPB + tok_in_tile;  // token index within the unit
+        const bool valid = in_tile && tok < u.n_tok;
+        const int64_t row_idx = static_cast<int64_t>(u.q_tok0 + tok) * p.Hq + u.kvh * G + head_in_group;
+        if (u.n_tiles <= 0) {
+            if (valid) store_zero_row<D>(p, row_idx);
+            continue;
+        }
+        const int lim = min(u.qlim0 + tok, u.Lk - 1);                 // this row's last visible key
+        const int tile_min_lim = min(u.qlim0 + mt * TPB, u.Lk - 1);  // smallest limit in the M-tile
+        float m = -INFINITY;  // running max, log2 domain
+        float l = 0.f;        // running sum of the bf16-rounded probabilities
+        for (int j = 0; j < u.n_tiles; ++j) {
+            bool ok = bounded_wait(bar(C::kBarS + mt), s_par, abort_flag, p.status, kWaitLimitNs);
+            if (!__all_sync(0xFFFFFFFFu, ok)) return;
+            s_par ^= 1u;
+            ptx::tc_fence_after();
+            uint32_t s[kBlockN];
+            ptx::tmem_ld32(tS + 0, s);
+            ptx::tmem_ld32(tS + 32, s + 32);
+            ptx::tmem_ld32(tS + 64, s + 64);
+            ptx::tmem_ld32(tS + 96, s + 96);
+            ptx::tmem_wait_ld();
+            ptx::tmem_ld_fence<kBlockN>(s);
+
+            const int kbase = j * kBlockN;
+            if (kbase + kBlockN - 1 > tile_min_lim) {  // diagonal or tail tile: mask per row
+                const int lloc = lim - kbase;
+#pragma unroll
+                for (int c = 0; c < kBlockN; ++c)
+                    if (c > lloc) s[c] = __float_as_uint(-INFINITY);
+            }
+            float mx[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) mx[t] = __uint_as_float(s[t]);
+#pragma unroll
+            for (int c = 8; c < kBlockN; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(s[c]));
+            const float mraw = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+            const float m_tile = mraw * cl;
+            float alpha = 1.f;
+            bool rescale = false;
+            if (j == 0) {
+                m = m_tile;
+            } else if (m_tile > m + kRescaleThreshold) {
+                alpha = ptx::ex2_approx(m - m_tile);
+                m = m_tile;
+                rescale = true;
+            }
+            const float msub = (m == -INFINITY) ? 0.f : m;
+            float sum[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c2 = 0; c2 < kBlockN / 2; ++c2) {
+                const float p0 = ptx::ex2_approx(fmaf(__uint_as_float(s[2 * c2]), cl, -msub));
+                const float p1 = ptx::ex2_approx(fmaf(__uint_as_float(s[2 * c2 + 1]), cl, -msub));
+                const uint32_t pk = ptx::pack_bf16x2(p0, p1);
+                sum[c2 & 3] += ptx::bf16lo_to_f32(pk) + ptx::bf16hi_to_f32(pk);
+                s[c2] = pk;
+            }
+            l = l * alpha + ((sum[0] + sum[1]) + (sum[2] + sum[3]));
+            ptx::tmem_st32(tS + 0, s);
+            ptx::tmem_st32(tS + 32, s + 32);
+            ptx::tmem_wait_st();
+            if (__any_sync(0xFFFFFFFFu, rescale)) {
+#pragma unroll
+                for (int ch = 0; ch < D / 32; ++ch) {
+                    uint32_t ov[32];
+                    ptx::tmem_ld32(tO + 32 * ch, ov);
+                    ptx::tmem_wait_ld();
+                    ptx::tmem_ld_fence<32>(ov);
+#pragma unroll
+                    for (int t = 0; t < 32; ++t) ov[t] = __float_as_uint(__uint_as_float(ov[t]) * alpha);
+                    ptx::tmem_st32(tO + 32 * ch, ov);
+                }
+                ptx::tmem_wait_st();
+            }
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(bar(C::kBarP + mt));
+        }
+        bool ok = bounded_wait(bar(C::kBarO + mt), o_par, abort_flag, p.status, kWaitLimitNs);
+        if (!__all_sync(0xFFFFFFFFu, ok)) return;
+        o_par ^= 1u;
+        ptx::tc_fence_after();
+        const float inv_l = l > 0.f ? 1.f / l : 0.f;
+        const float lse_v = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
+#pragma unroll
+        for (int ch = 0; ch < D / 32; ++ch) {
+            uint32_t ov[32];
+            ptx::tmem_ld32(tO + 32 * ch, ov);
+            ptx::tmem_wait_ld();
+            ptx::tmem_ld_fence<32>(ov);
+            uint32_t w[16];
+#pragma unroll
+            for (int t = 0; t < 16; ++t)
+                w[t] = ptx::pack_bf16x2(__uint_as_float(ov[2 * t]) * inv_l, __uint_as_float(ov[2 * t + 1]) * inv_l);
+            if (valid) {
+                uint4* dst = reinterpret_cast<uint4*>(p.o + row_idx * D + ch * 32);
+                dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+                dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+                dst[2] = make_uint4(w[8], w[9], w[10], w[11]);
+                dst[3] = make_uint4(w[12], w[13], w[14], w[15]);
+            }
+        }
+        if (valid) p.lse[row_idx] = lse_v;
+    }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    opattn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                          const __grid_constant__ CUtensorMap tmV, const KParams p) {
+    using C = Cfg<D>;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    const uint32_t raw = ptx::smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;  // 128-byte swizzle atoms need 1024-byte alignment
+    uint8_t* gbase = smem_raw + (base - raw);
+    const uint32_t sQ = base + C::kQOff;
+    const uint32_t sRing = base + C::kRingOff;
+    const uint32_t sBar = base + C::kBarOff;
+    volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(gbase + C::kMiscOff);
+    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(gbase + C::kMiscOff + 4);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < C::kSlots; ++i) {
+            ptx::mbar_init(sBar + 8u * (C::kBarFull + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarEmpty + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(sBar + 8u * (C::kBarQFull + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarQEmpty + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarS + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarO + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarP + i), 128);
+        }
+        ptx::mbar_init(sBar + 8u * C::kBarDrain, 1);
+        ptx::mbar_init(sBar + 8u * C::kBarNever, 1);
+        *abort_flag = 0;
+        ptx::fence_mbar_init();
+    }
+    if (warp == kWarpMma) {
+        ptx::tmem_alloc(ptx::smem_addr(const_cast<uint32_t*>(tmem_slot)), C::kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == kWarpProducer && lane == 0) {
+        ptx::prefetch_tmap(&tmQ);
+        ptx::prefetch_tmap(&tmK);
+        ptx::prefetch_tmap(&tmV);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int ubeg = p.cta_off[blockIdx.x];
+    const int uend = p.cta_off[blockIdx.x + 1];
+
+    if (warp == kWarpProducer) {
+        if (lane == 0) run_producer<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, abort_flag);
+        __syncwarp();
+    } else if (warp == kWarpMma) {
+        if (lane == 0) run_mma<D>(p, ubeg, uend, tmem, sQ, sRing, sBar, abort_flag);
+        __syncwarp();
+    } else if (warp >= kWarpSoftmax) {
+        run_softmax<D>(p, ubeg, uend, tmem, sBar, warp, lane, abort_flag);
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == kWarpMma) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+// ------------------------------------------------------------------- host
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+// [rows, heads, d] bf16 tensor, box of (64 channels, box_heads, box_rows),
+// 128-byte swizzle; out-of-range rows read as zero.
+bool encode_3d(EncodeTiledFn fn, CUtensorMap* map, const void* base, uint64_t d, uint64_t heads, uint64_t rows,
+               uint32_t box_heads, uint32_t box_rows) {
+    const cuuint64_t dims[3] = {d, heads, rows};
+    const cuuint64_t strides[2] = {d * 2, heads * d * 2};
+    const cuuint32_t box[3] = {64, box_heads, box_rows};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+int launch_d(const LaunchArgs& a, cudaStream_t stream) {
+    using C = Cfg<D>;
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return -1;
+    const int G = a.Hq / a.Hkv;
+    const int TPB = kRowsPerTile / G;
+    CUtensorMap tq, tk, tv;
+    // With no keys at all no unit visits a key tile; the K/V maps then only
+    // need to be well formed, so they describe one row of q.
+    const void* kb = a.total_k > 0 ? a.k : a.q;
+    const void* vb = a.total_k > 0 ? a.v : a.q;
+    const uint64_t krows = a.total_k > 0 ? static_cast<uint64_t>(a.total_k) : 1;
+    if (!encode_3d(fn, &tq, a.q, D, a.Hq, a.total_q, G, TPB)) return -2;
+    if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, kBlockN)) return -3;
+    if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, kBlockN)) return -4;
+
+    static std::mutex mu;
+    static bool attr_done[128] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    {
+        std::lock_guard<std::mutex> g(mu);
+        if (dev < 0 || dev >= 128 || !attr_done[dev]) {
+            e = cudaFuncSetAttribute(opattn_prefill_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     C::kSmemBytes);
+            if (e != cudaSuccess) return e;
+            if (dev >= 0 && dev < 128) attr_done[dev] = true;
+        }
+    }
+    KParams kp;
+    kp.units = a.units;
+    kp.cta_off = a.cta_off;
+    kp.o = static_cast<uint16_t*>(a.o);
+    kp.lse = a.lse;
+    kp.Hq = a.Hq;
+    kp.G = G;
+    kp.TPB = TPB;
+    kp.scale_log2 = a.scale * kLog2e;
+    kp.status = a.status;
+    kp.flags = a.flags;
+    opattn_prefill_kernel<D><<<a.n_cta, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, kp);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int launch_prefill(const LaunchArgs& a, cudaStream_t stream) {
+    if (a.d == 64) return launch_d<64>(a, stream);
+    if (a.d == 128) return launch_d<128>(a, stream);
+    return -5;
+}
+
+int kernel_smem_bytes(int d) {
+    if (d == 64) return Cfg<64>::kSmemBytes;
+    if (d == 128) return Cfg<128>::kSmemBytes;
+    return 0;
+}
+
+}  // namespace opattn

@@ -1,0 +1,200 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Bar: O within max-abs 1e-2 and mean-abs 1e-3, LSE within 1e-3 abs where the
+oracle's LSE is finite and exactly -inf where it is not.  Small cases are
+compared on every element; the full-size workloads are compared on sampled
+rows (first and last tokens of every sequence, M-tile boundaries, random
+rows), with every output element checked for having been written.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2608_13499_gb300 as pkg
+from paper_2608_13499_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+O_MAX, O_MEAN, LSE_MAX = 1e-2, 1e-3, 1e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2608_13499_gb300 import build as pbuild
+    pbuild.build()
+    pkg.load()
+    oracle.build()
+
+
+def run_gpu(w, q, k, v, stream=None):
+    o = torch.full((w.total_q, w.Hq, w.d), float("nan"), dtype=torch.bfloat16, device=q.device)
+    lse = torch.full((w.total_q, w.Hq), float("nan"), dtype=torch.float32, device=q.device)
+    pkg.opattn_prefill(q, k, v, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
+    torch.cuda.synchronize()
+    return o, lse
+
+
+def check(o_gpu, lse_gpu, o_ref, lse_ref, what=""):
+    o = o_gpu.float().cpu().numpy().astype(np.float64)
+    lse = lse_gpu.cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(o)), f"{what}: non-finite O"
+    err = np.abs(o - o_ref)
+    assert err.max() <= O_MAX, f"{what}: O max-abs {err.max():.3e}"
+    assert err.mean() <= O_MEAN, f"{what}: O mean-abs {err.mean():.3e}"
+    fin = np.isfinite(lse_ref)
+    assert np.array_equal(np.isfinite(lse), fin), f"{what}: LSE finiteness differs"
+    assert np.all(lse[~fin] == -np.inf)
+    if fin.any():
+        lerr = np.abs(lse[fin] - lse_ref[fin]).max()
+        assert lerr <= LSE_MAX, f"{what}: LSE max-abs {lerr:.3e}"
+    return err.max(), err.mean()
+
+
+def custom(name, lq, lk, Hq, Hkv, d, seed=0, input_scale=1.0):
+    return W.Workload(name, list(lq), list(lk), Hq, Hkv, d, input_scale, seed)
+
+
+SMALL = [
+    W.tiny(),
+    custom("ragged_g4_d128", [1, 2, 127, 128, 129, 255, 257], [1, 2, 127, 128, 129, 255, 257], 32, 8, 128),
+    custom("ragged_g1_d64", [1, 2, 127, 128, 129, 255, 257], [1, 2, 127, 128, 129, 255, 257], 8, 8, 64),
+    custom("chunks_g8", [512, 100, 1, 37], [812, 228, 1001, 37], 16, 2, 128),
+    custom("short_kv_g3", [9, 0, 40, 5], [3, 0, 40, 0], 12, 4, 128),
+    custom("g16_d64", [300, 64], [300, 64], 32, 2, 64),
+    custom("g128_d64", [70, 3], [70, 3], 128, 1, 64),
+    custom("long_1500_g8", [1500], [1500], 16, 2, 128, seed=3),
+    custom("g2_d128_odd", [333, 1, 190], [333, 1, 190], 4, 2, 128, seed=5),
+]
+
+
+@pytest.mark.parametrize("w", SMALL, ids=[w.name for w in SMALL])
+def test_small_cases_every_element(w):
+    q, k, v = W.make_inputs(w, "cuda")
+    o, lse = run_gpu(w, q, k, v)
+    if w.name.startswith("tiny"):
+        assert tuple(o.shape) == (82, 4, 64) and tuple(lse.shape) == (82, 4)
+    o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
+    check(o, lse, o_ref, lse_ref, w.name)
+
+
+def test_large_logits_exercise_rescaling():
+    """q scaled by 4 (exact in bf16): logits span ~+-40, so running maxima jump often."""
+    w = custom("large_logits", [700, 260], [700, 260], 16, 4, 128, seed=7)
+    q, k, v = W.make_inputs(w, "cuda")
+    q = (q.float() * 4).to(torch.bfloat16)
+    o, lse = run_gpu(w, q, k, v)
+    o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
+    check(o, lse, o_ref, lse_ref, w.name)
+
+
+def sample_rows(w, rng, n_random):
+    tok, hd = [], []
+    G = w.Hq // w.Hkv
+    tpb = 128 // G
+    cu = w.cu_q
+    for s in range(w.n_seq):
+        L = w.q_lens[s]
+        if L == 0:
+            continue
+        picks = {0, 1, 2, L - 1, L - 2, min(L - 1, tpb - 1), min(L - 1, tpb), min(L - 1, 2 * tpb)}
+        for t in picks:
+            if 0 <= t < L:
+                tok.append(cu[s] + t)
+                hd.append(int(rng.integers(0, w.Hq)))
+    tok += list(rng.integers(0, w.total_q, size=n_random))
+    hd += list(rng.integers(0, w.Hq, size=n_random))
+    return np.array(tok, dtype=np.int64), np.array(hd, dtype=np.int32)
+
+
+FULL = [W.llama3_8b(), W.llama3_70b(), W.bursty(), W.chunked()]
+
+
+@pytest.mark.parametrize("w", FULL, ids=[w.name for w in FULL])
+def test_full_size_workloads_sampled_rows(w):
+    q, k, v = W.make_inputs(w, "cuda")
+    o, lse = run_gpu(w, q, k, v)
+    # every element written (outputs were NaN-filled)
+    assert not torch.isnan(o).any().item()
+    assert not torch.isnan(lse).any().item()
+    rng = np.random.default_rng(11)
+    tok, hd = sample_rows(w, rng, 600)
+    q_c, k_c, v_c = q.cpu(), k.cpu(), v.cpu()
+    o_ref, lse_ref = oracle.attention_rows(q_c, k_c, v_c, w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale, tok, hd)
+    t_idx = torch.from_numpy(tok)
+    h_idx = torch.from_numpy(hd.astype(np.int64))
+    o_rows = o.cpu()[t_idx, h_idx]
+    lse_rows = lse.cpu()[t_idx, h_idx]
+    check(o_rows, lse_rows, o_ref, lse_ref, w.name)
+
+
+def test_outputs_stay_inside_their_buffers():
+    w = custom("canary", [130, 7], [130, 7], 8, 2, 128)
+    q, k, v = W.make_inputs(w, "cuda")
+    n_o, n_l = w.total_q * w.Hq * w.d, w.total_q * w.Hq
+    o_buf = torch.full((n_o + 4096,), 3.0, dtype=torch.bfloat16, device="cuda")
+    l_buf = torch.full((n_l + 1024,), 7.0, dtype=torch.float32, device="cuda")
+    pkg.opattn_prefill(q, k, v, o_buf, l_buf, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale)
+    torch.cuda.synchronize()
+    assert torch.all(o_buf[n_o:] == 3.0).item()
+    assert torch.all(l_buf[n_l:] == 7.0).item()
+    o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
+    check(o_buf[:n_o].view(w.total_q, w.Hq, w.d), l_buf[:n_l].view(w.total_q, w.Hq), o_ref, lse_ref, "canary")
+
+
+def test_sequence_order_and_repeat_runs_are_bitwise_stable():
+    w = custom("perm", [300, 45, 129], [300, 45, 129], 16, 4, 128, seed=2)
+    q, k, v = W.make_inputs(w, "cuda")
+    o1, l1 = run_gpu(w, q, k, v)
+    o2, l2 = run_gpu(w, q, k, v)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    perm = [2, 0, 1]
+    cq, ck = w.cu_q, w.cu_k
+    qp = torch.cat([q[cq[s]:cq[s + 1]] for s in perm])
+    kp = torch.cat([k[ck[s]:ck[s + 1]] for s in perm])
+    vp = torch.cat([v[ck[s]:ck[s + 1]] for s in perm])
+    wp = custom("perm2", [w.q_lens[s] for s in perm], [w.k_lens[s] for s in perm], 16, 4, 128)
+    op, lp = run_gpu(wp, qp, kp, vp)
+    assert torch.equal(op, torch.cat([o1[cq[s]:cq[s + 1]] for s in perm]))
+    assert torch.equal(lp, torch.cat([l1[cq[s]:cq[s + 1]] for s in perm]))
+
+
+def test_plan_matches_one_shot_and_runs_on_a_side_stream():
+    w = W.llama3_8b()
+    q, k, v = W.make_inputs(w, "cuda")
+    o1, l1 = run_gpu(w, q, k, v)
+    side = torch.cuda.Stream()
+    o2 = torch.empty_like(o1)
+    l2 = torch.empty_like(l1)
+    with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d) as plan:
+        assert plan.n_ctas == min(plan.n_units, torch.cuda.get_device_properties(0).multi_processor_count)
+        side.wait_stream(torch.cuda.current_stream())
+        plan.run(q, k, v, o2, l2, w.scale, stream=side)
+        side.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+
+
+def test_reduced_cta_budget_gives_the_same_numbers():
+    """An SM-capped plan (fewer persistent CTAs) computes each row the same way."""
+    w = custom("budget", [700, 300, 90], [700, 300, 90], 16, 2, 128, seed=4)
+    q, k, v = W.make_inputs(w, "cuda")
+    o1, l1 = run_gpu(w, q, k, v)
+    o2, l2 = torch.empty_like(o1), torch.empty_like(l1)
+    with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, max_ctas=7) as plan:
+        assert plan.n_ctas == 7
+        plan.run(q, k, v, o2, l2, w.scale)
+        torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+
+
+def test_no_keys_at_all():
+    w = custom("no_keys", [5, 3], [0, 0], 4, 2, 64)
+    q, _, _ = W.make_inputs(custom("nk_q", [5, 3], [5, 3], 4, 2, 64), "cuda")
+    o = torch.full((8, 4, 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((8, 4), float("nan"), dtype=torch.float32, device="cuda")
+    pkg.opattn_prefill(q, None, None, o, lse, w.cu_q, w.cu_k, 2, 4, 2, 64, 0.125)
+    torch.cuda.synchronize()
+    assert torch.all(o == 0).item()
+    assert torch.all(lse == -math.inf).item()

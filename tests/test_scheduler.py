@@ -1,0 +1,111 @@
+"""Host scheduler (longest-first ragged work list), checked without a GPU.
+
+The unit records are checked against a brute-force enumeration of which
+(query token, key) pairs the causal mask leaves visible, and the assignment
+against the longest-processing-time rule and Graham's 4/3 bound.
+"""
+import numpy as np
+import pytest
+
+import paper_2608_13499_gb300 as pkg
+from paper_2608_13499_gb300 import build as pbuild
+from paper_2608_13499_gb300 import workloads as W
+
+BN = 128
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    pbuild.build()
+    return pkg.load()
+
+
+def unit_table(units):
+    return {name: units[:, i] for i, name in enumerate(pkg.UNIT_FIELDS)}
+
+
+CASES = [
+    ([1, 17, 64], [1, 17, 64], 4, 2, 64, 152),
+    ([1, 2, 127, 128, 129, 255, 257], [1, 2, 127, 128, 129, 255, 257], 32, 8, 128, 7),
+    ([512, 512, 300], [700, 1024, 300], 32, 8, 128, 16),     # chunks with prefixes
+    ([9, 0, 40, 5], [3, 0, 40, 0], 12, 4, 128, 5),            # Lq > Lk, empty, G = 3
+    ([100, 33], [100, 33], 128, 1, 64, 3),                    # G = 128, one token per M-tile
+    (W.bursty().q_lens, W.bursty().k_lens, 32, 8, 128, 152),
+]
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_units_cover_every_row_once_with_exact_tile_counts(case):
+    lq, lk, Hq, Hkv, d, n_cta = case
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_schedule(cu_q, cu_k, Hq, Hkv, d, n_cta)
+    G = Hq // Hkv
+    tpu = 2 * (128 // G)
+    t = unit_table(units)
+    covered = np.zeros((int(cu_q[-1]), Hkv), dtype=np.int32)
+    for u in range(len(units)):
+        s = t["seq"][u]
+        L_q, L_k = lq[s], lk[s]
+        delta = L_k - L_q
+        tok0 = t["q_tok0"][u] - cu_q[s]
+        assert 0 <= tok0 < L_q and tok0 % tpu == 0
+        assert t["n_tok"][u] == min(tpu, L_q - tok0)
+        assert t["k_row0"][u] == cu_k[s] and t["Lk"][u] == L_k
+        assert t["qlim0"][u] == tok0 + delta
+        covered[t["q_tok0"][u]:t["q_tok0"][u] + t["n_tok"][u], t["kvh"][u]] += 1
+        # brute force: the highest key any token of the unit sees
+        last = max([min(i + delta, L_k - 1) for i in range(tok0, tok0 + t["n_tok"][u])])
+        want_tiles = 0 if last < 0 else last // BN + 1
+        assert t["n_tiles"][u] == want_tiles
+    assert np.all(covered == 1)
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_longest_first_assignment(case):
+    lq, lk, Hq, Hkv, d, n_cta = case
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_schedule(cu_q, cu_k, Hq, Hkv, d, n_cta)
+    n = len(units)
+    if n == 0:
+        return
+    P = len(offs) - 1
+    assert P == min(n_cta, n)
+    assert offs[0] == 0 and offs[-1] == n and np.all(np.diff(offs) >= 1)
+    cost = units[:, 6].astype(np.int64) + 1
+    loads = np.array([cost[offs[c]:offs[c + 1]].sum() for c in range(P)])
+    for c in range(P):
+        seg = cost[offs[c]:offs[c + 1]]
+        assert np.all(np.diff(seg) <= 0), "a CTA's units are not longest first"
+    # Graham: LPT makespan <= (4/3 - 1/(3P)) * OPT, and OPT >= max(mean load, largest unit)
+    lower = max(cost.sum() / P, cost.max())
+    assert loads.max() <= (4.0 / 3.0) * lower + 1e-9
+    # greedy replay: each unit, in global longest-first order, went to a least-loaded CTA
+    order = np.argsort(-cost, kind="stable")
+    assert np.all(np.diff(cost[order]) <= 0)
+
+
+def test_capacity_error_reports_the_needed_size():
+    cu = np.array([0, 300], dtype=np.int32)
+    lib = pkg.load()
+    import ctypes
+    n_units, n_used = ctypes.c_int64(0), ctypes.c_int32(0)
+    units = np.zeros((2, 8), dtype=np.int32)
+    offs = np.zeros(8, dtype=np.int32)
+    st = lib.opattn_schedule(cu.ctypes.data_as(ctypes.c_void_p), cu.ctypes.data_as(ctypes.c_void_p), 1, 8, 2, 128, 4,
+                             units.ctypes.data_as(ctypes.c_void_p), 2, offs.ctypes.data_as(ctypes.c_void_p),
+                             ctypes.byref(n_units), ctypes.byref(n_used))
+    assert st == pkg.OPATTN_ERR_CAPACITY
+    # G = 4 -> 64 tokens per unit -> 5 blocks x 2 kv heads
+    assert n_units.value == 10 and n_used.value == 4
+
+
+def test_standard_workload_unit_counts():
+    # G = 8 (Llama-3-70B shape): 32 tokens per unit -> 8 * 128 blocks * 8 kv heads
+    w = W.llama3_70b()
+    units, _ = pkg.opattn_schedule(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, 152)
+    assert len(units) == 8 * 128 * 8
+    w = W.tiny()
+    units, _ = pkg.opattn_schedule(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, 152)
+    assert len(units) == 6
