@@ -324,7 +324,8 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
         const int lim = min(u.qlim0 + tok, u.Lk - 1);                 // this row's last visible key
         const int tile_min_lim = min(u.qlim0 + mt * TPB, u.Lk - 1);  // smallest limit in the M-tile
         float m = -INFINITY;  // running max, log2 domain
-        float l = 0.f;        // running sum of the bf16-rounded probabilities
+        float l = 0.f;        // running sum of the probabilities (fp32, for LSE)
+        float lh = 0.f;       // running sum of the bf16-rounded probabilities PV consumes (normalises O)
         for (int j = 0; j < u.n_tiles; ++j) {
             bool ok = bounded_wait(bar(C::kBarS + mt), s_par, abort_flag, p.status, kWaitLimitNs);
             if (!__all_sync(0xFFFFFFFFu, ok)) return;
@@ -364,15 +365,18 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
             }
             const float msub = (m == -INFINITY) ? 0.f : m;
             float sum[4] = {0.f, 0.f, 0.f, 0.f};
+            float sumh[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int c2 = 0; c2 < kBlockN / 2; ++c2) {
                 const float p0 = ptx::ex2_approx(fmaf(__uint_as_float(s[2 * c2]), cl, -msub));
                 const float p1 = ptx::ex2_approx(fmaf(__uint_as_float(s[2 * c2 + 1]), cl, -msub));
                 const uint32_t pk = ptx::pack_bf16x2(p0, p1);
-                sum[c2 & 3] += ptx::bf16lo_to_f32(pk) + ptx::bf16hi_to_f32(pk);
+                sum[c2 & 3] += p0 + p1;
+                sumh[c2 & 3] += ptx::bf16lo_to_f32(pk) + ptx::bf16hi_to_f32(pk);
                 s[c2] = pk;
             }
             l = l * alpha + ((sum[0] + sum[1]) + (sum[2] + sum[3]));
+            lh = lh * alpha + ((sumh[0] + sumh[1]) + (sumh[2] + sumh[3]));
             ptx::tmem_st32(tS + 0, s);
             ptx::tmem_st32(tS + 32, s + 32);
             ptx::tmem_wait_st();
@@ -396,7 +400,9 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
         if (!__all_sync(0xFFFFFFFFu, ok)) return;
         o_par ^= 1u;
         ptx::tc_fence_after();
-        const float inv_l = l > 0.f ? 1.f / l : 0.f;
+        // O is normalised by the sum of the same rounded weights the PV MMA
+        // used (a weighted mean of V rows); LSE uses the unrounded sum.
+        const float inv_l = lh > 0.f ? 1.f / lh : 0.f;
         const float lse_v = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
 #pragma unroll
         for (int ch = 0; ch < D / 32; ++ch) {
