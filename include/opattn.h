@@ -90,6 +90,35 @@ OPATTN_API opattn_status opattn_prefill(const void *q, const void *k, const void
                              void *stream);
 
 /*
+ * Allocation-free variant of opattn_prefill (the paper has no counterpart;
+ * this is a library convenience).  For callers that cannot have the library
+ * allocate device memory: a serving engine that reserves almost all of HBM
+ * for its KV cache and hands out memory only from its own pool, a process
+ * whose device memory is capped by a quota, or a device without the
+ * stream-ordered allocator.  Same arguments, computation and asynchrony as
+ * opattn_prefill; the caller still provides q, k, v, o and lse.  The work
+ * list and status word go to a fixed device array inside the library
+ * (OPATTN_NOALLOC_MAX_UNITS work units of 32 bytes plus 8 KiB, about 1 MiB),
+ * which every GPU that loads the library keeps until the process exits.  It
+ * calls no cudaMalloc, cudaMallocAsync or cudaFree (the host side builds
+ * the list in ordinary heap memory and copies it with cudaMemcpyAsync).
+ *   - The first call on a device looks up the array's device address with
+ *     that device current; make that first call before any stream capture.
+ *   - All calls share the one array and each overwrites it: calls that
+ *     overlap on the GPU (unordered streams, or several host threads) race,
+ *     so order them on one stream or serialize them.
+ *   - Returns OPATTN_ERR_CAPACITY, before touching the GPU, when the batch
+ *     needs more than OPATTN_NOALLOC_MAX_UNITS work units (a unit is one kv
+ *     head x 2 * (128 / G) query tokens of one sequence); use
+ *     opattn_prefill for such batches.
+ */
+#define OPATTN_NOALLOC_MAX_UNITS 32768
+OPATTN_API opattn_status opattn_prefill_noalloc(const void *q, const void *k, const void *v, void *o, float *lse,
+                                                const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                                                int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
+                                                void *stream);
+
+/*
  * Diagnostic variant: the same computation, then it synchronizes `stream`
  * and reads back the kernel's status word; returns OPATTN_ERR_TIMEOUT if a
  * bounded wait expired.  `flags` must be 0 except in the library's own

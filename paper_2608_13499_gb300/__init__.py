@@ -24,6 +24,7 @@ OPATTN_ERR_CUDA = 4
 OPATTN_ERR_TIMEOUT = 5
 OPATTN_ERR_CAPACITY = 6
 OPATTN_FLAG_TEST_FORCE_TIMEOUT = 1
+OPATTN_NOALLOC_MAX_UNITS = 32768
 
 UNIT_FIELDS = ("q_tok0", "n_tok", "k_row0", "Lk", "qlim0", "kvh", "n_tiles", "seq")
 
@@ -54,6 +55,8 @@ def load():
             lib.opattn_status_string.argtypes = [i32]
             lib.opattn_prefill.restype = ctypes.c_int
             lib.opattn_prefill.argtypes = [P, P, P, P, P, P, P, i32, i32, i32, i32, f32, P]
+            lib.opattn_prefill_noalloc.restype = ctypes.c_int
+            lib.opattn_prefill_noalloc.argtypes = [P, P, P, P, P, P, P, i32, i32, i32, i32, f32, P]
             lib.opattn_prefill_checked.restype = ctypes.c_int
             lib.opattn_prefill_checked.argtypes = [P, P, P, P, P, P, P, i32, i32, i32, i32, f32, P, u32]
             lib.opattn_plan_create.restype = ctypes.c_int
@@ -115,6 +118,22 @@ def opattn_prefill(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: int, Hq: 
                                int(n_seq), int(Hq), int(Hkv), int(d), float(scale), _stream_handle(stream))
     if check and st != OPATTN_OK:
         raise OpattnError(st, "opattn_prefill")
+    return st
+
+
+def opattn_prefill_noalloc(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int,
+                           scale: float, stream=None, *, check: bool = True) -> int:
+    """C ``opattn_prefill_noalloc``: same arguments as opattn_prefill, but the library
+    allocates no device memory (its work list goes to a fixed ~1 MiB device array
+    shared by all calls; see include/opattn.h).  For callers that cannot let a
+    library allocate, e.g. an engine that has reserved nearly all HBM for its own
+    pool.  Calls that overlap on the GPU race on the shared array."""
+    cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
+    st = load().opattn_prefill_noalloc(_dptr(q), _dptr(k), _dptr(v), _dptr(o), _dptr(lse), _np_ptr(cq),
+                                       _np_ptr(ck), int(n_seq), int(Hq), int(Hkv), int(d), float(scale),
+                                       _stream_handle(stream))
+    if check and st != OPATTN_OK:
+        raise OpattnError(st, "opattn_prefill_noalloc")
     return st
 
 

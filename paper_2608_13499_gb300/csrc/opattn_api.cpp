@@ -294,6 +294,53 @@ opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o,
     return OPATTN_OK;
 }
 
+static_assert(kNoAllocMaxUnits == OPATTN_NOALLOC_MAX_UNITS, "opattn.h and the scratch size disagree");
+
+// Work units of a batch without building the schedule (same enumeration
+// as build_schedule).
+int64_t count_units(const int32_t* cu_q, const Geometry& g) {
+    const int64_t tpu = 2 * g.TPB;
+    int64_t n = 0;
+    for (int32_t s = 0; s < g.n_seq; ++s) n += (static_cast<int64_t>(cu_q[s + 1] - cu_q[s]) + tpu - 1) / tpu;
+    return n * g.Hkv;
+}
+
+// Same computation as prefill_impl with the work list in the library's
+// fixed device array: nothing is allocated on the device.
+opattn_status prefill_noalloc_impl(const void* q, const void* k, const void* v, void* o, float* lse,
+                                   const int32_t* cu_q, const int32_t* cu_k, int32_t n_seq, int32_t Hq,
+                                   int32_t Hkv, int32_t d, float scale, cudaStream_t stream) {
+    Geometry g;
+    opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    if (g.total_q == 0) return OPATTN_OK;
+    st = check_tensors(q, k, v, o, lse, scale, g);
+    if (st != OPATTN_OK) return st;
+    if (count_units(cu_q, g) > kNoAllocMaxUnits) return OPATTN_ERR_CAPACITY;
+    const int sms = device_sm_count();
+    if (sms <= 0) return OPATTN_ERR_CUDA;
+
+    Schedule sch;
+    build_schedule(cu_q, cu_k, g, std::min(sms, kNoAllocMaxCtas), &sch);
+    const WorkLayout w = work_layout(sch);
+    void* scratch = nullptr;
+    size_t scratch_bytes = 0;
+    if (noalloc_scratch(&scratch, &scratch_bytes) != 0) return OPATTN_ERR_CUDA;
+    if (w.bytes > scratch_bytes) return OPATTN_ERR_CAPACITY;
+    // The list is copied from ordinary (pageable) host memory: the runtime
+    // stages it before cudaMemcpyAsync returns, so the vector may go away.
+    std::vector<uint8_t> host(w.upload_bytes);
+    pack_upload(sch, w, host.data());
+    uint8_t* work = static_cast<uint8_t*>(scratch);
+    if (cudaMemcpyAsync(work, host.data(), w.upload_bytes, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return OPATTN_ERR_CUDA;
+    // The array keeps the previous call's contents: the status word must
+    // start at zero.
+    if (cudaMemsetAsync(work + w.off_status, 0, sizeof(int32_t), stream) != cudaSuccess) return OPATTN_ERR_CUDA;
+    const LaunchArgs a = make_args(q, k, v, o, lse, g, scale, work, w, sch.n_cta, 0u);
+    return launch_prefill(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+}
+
 }  // namespace
 }  // namespace opattn
 
@@ -329,6 +376,13 @@ opattn_status opattn_prefill(const void* q, const void* k, const void* v, void* 
                              int32_t Hkv, int32_t d, float scale, void* stream) {
     return prefill_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
                         static_cast<cudaStream_t>(stream), 0u, false);
+}
+
+opattn_status opattn_prefill_noalloc(const void* q, const void* k, const void* v, void* o, float* lse,
+                                     const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
+                                     int32_t Hq, int32_t Hkv, int32_t d, float scale, void* stream) {
+    return prefill_noalloc_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
+                                static_cast<cudaStream_t>(stream));
 }
 
 opattn_status opattn_prefill_checked(const void* q, const void* k, const void* v, void* o, float* lse,

@@ -56,6 +56,15 @@ struct LaunchArgs {
     uint32_t flags;
 };
 
+// Limits of the allocation-free entry point (opattn_prefill_noalloc), whose
+// work list lives in a fixed device array (opattn_noalloc.cu).
+constexpr int64_t kNoAllocMaxUnits = 32768;
+constexpr int32_t kNoAllocMaxCtas = 1024;
+// Implemented in opattn_noalloc.cu: device address and size of that array on
+// the current device (looked up on the first call per device).  Returns a
+// cudaError_t as int.
+int noalloc_scratch(void** ptr, size_t* bytes);
+
 // Implemented in opattn_kernel.cu.  Returns a cudaError_t (as int) or a
 // negative value when the tensor maps cannot be encoded.
 int launch_prefill(const LaunchArgs& a, cudaStream_t stream);
