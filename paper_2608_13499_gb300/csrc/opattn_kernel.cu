@@ -52,6 +52,16 @@ constexpr uint64_t kDrainLimitNs = 200000000ull;  // in-flight copies / MMAs aft
 // probabilities stay below 2^8, far inside bf16 and fp32 range.
 constexpr float kRescaleThreshold = 8.0f;
 constexpr float kLn2 = 0.693147180559945309f;
+// Register split: the kernel is compiled for 168 registers per thread at
+// launch (384 threads, one CTA per SM = 64512 registers).  Warpgroup 0
+// (producer, MMA, two idle warps) gives registers back, the two softmax
+// warpgroups take them: 104 * 128 + 200 * 256 = 168 * 384.  The host refuses
+// to launch a build whose register count differs, because a split larger
+// than the launch total would make setmaxnreg.inc wait forever.
+constexpr int kLaunchRegs = 168;
+constexpr uint32_t kRegsControl = 104;
+constexpr uint32_t kRegsSoftmax = 200;
+static_assert(kRegsControl * 128 + kRegsSoftmax * 256 == kLaunchRegs * kThreads, "register split");
 constexpr float kLog2e = 1.442695040888963407f;
 
 template <int D>
@@ -60,7 +70,7 @@ struct Cfg {
     static constexpr int kDBlocks = D / 64;                        // 128-byte swizzle column blocks
     static constexpr int kQTileBytes = kRowsPerTile * D * 2;       // one M-tile of Q
     static constexpr int kSlotBytes = kBlockN * D * 2;             // one K or V tile
-    static constexpr int kSlots = D == 128 ? 4 : 8;                // ring depth (K and V alternate)
+    static constexpr int kSlots = D == 128 ? 5 : 12;               // ring depth (K and V alternate)
     static constexpr int kQOff = 0;
     static constexpr int kRingOff = 2 * kQTileBytes;
     static constexpr int kBarOff = kRingOff + kSlots * kSlotBytes;
@@ -130,6 +140,8 @@ __device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUten
     using C = Cfg<D>;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
     const uint32_t q_tx = static_cast<uint32_t>(p.G * p.TPB) * C::kQTxBytesPerRow;
+    const uint64_t keep = ptx::policy_evict_last();    // K/V tiles are re-read by other q blocks
+    const uint64_t stream = ptx::policy_evict_first();  // each Q tile is read once
     uint32_t slot = 0, ring_par = 0;
     uint32_t q_issued[2] = {0u, 0u};
     uint32_t ring_issued = 0;
@@ -146,8 +158,9 @@ __device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUten
             ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + i), q_tx);
 #pragma unroll
             for (int b = 0; b < C::kDBlocks; ++b)
-                ptx::tma_load_3d(sQ + i * C::kQTileBytes + b * (kRowsPerTile * 128), tmQ,
-                                 bar(C::kBarQFull + i), b * 64, u.kvh * p.G, u.q_tok0 + i * p.TPB);
+                ptx::tma_load_3d_hint(sQ + i * C::kQTileBytes + b * (kRowsPerTile * 128), tmQ,
+                                      bar(C::kBarQFull + i), b * 64, u.kvh * p.G, u.q_tok0 + i * p.TPB,
+                                      stream);
             ++q_issued[i];
         }
         for (int j = 0; j < u.n_tiles && !aborted; ++j) {
@@ -160,8 +173,8 @@ __device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUten
                 ptx::mbar_arrive_expect_tx(bar(C::kBarFull + slot), C::kSlotBytes);
 #pragma unroll
                 for (int b = 0; b < C::kDBlocks; ++b)
-                    ptx::tma_load_3d(sRing + slot * C::kSlotBytes + b * (kBlockN * 128), kv ? tmV : tmK,
-                                     bar(C::kBarFull + slot), b * 64, u.kvh, u.k_row0 + j * kBlockN);
+                    ptx::tma_load_3d_hint(sRing + slot * C::kSlotBytes + b * (kBlockN * 128), kv ? tmV : tmK,
+                                          bar(C::kBarFull + slot), b * 64, u.kvh, u.k_row0 + j * kBlockN, keep);
                 ++ring_issued;
                 if (++slot == C::kSlots) {
                     slot = 0;
@@ -346,13 +359,18 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
                 for (int c = 0; c < kBlockN; ++c)
                     if (c > lloc) s[c] = __float_as_uint(-INFINITY);
             }
+            // row max: 8 independent chains of 16 scores, 3-input max
             float mx[8];
 #pragma unroll
-            for (int t = 0; t < 8; ++t) mx[t] = __uint_as_float(s[t]);
+            for (int t = 0; t < 8; ++t) {
+                const uint32_t* v = s + 16 * t;
+                float a = ptx::max3f(__uint_as_float(v[0]), __uint_as_float(v[1]), __uint_as_float(v[2]));
 #pragma unroll
-            for (int c = 8; c < kBlockN; ++c) mx[c & 7] = fmaxf(mx[c & 7], __uint_as_float(s[c]));
-            const float mraw = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+                for (int i = 3; i < 15; i += 2) a = ptx::max3f(a, __uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+                mx[t] = fmaxf(a, __uint_as_float(v[15]));
+            }
+            const float mraw = ptx::max3f(ptx::max3f(mx[0], mx[1], mx[2]), ptx::max3f(mx[3], mx[4], mx[5]),
+                                          fmaxf(mx[6], mx[7]));
             const float m_tile = mraw * cl;
             float alpha = 1.f;
             bool rescale = false;
@@ -364,19 +382,35 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
                 rescale = true;
             }
             const float msub = (m == -INFINITY) ? 0.f : m;
-            float sum[4] = {0.f, 0.f, 0.f, 0.f};
-            float sumh[4] = {0.f, 0.f, 0.f, 0.f};
+            // p = 2^(s*c - m) on pairs: one packed FMA, two ex2, one bf16x2
+            // pack, two packed adds (exact and rounded running sums)
+            const uint64_t cc2 = ptx::f32x2(cl, cl);
+            const uint64_t nm2 = ptx::f32x2(-msub, -msub);
+            uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};   // (0.f, 0.f) pairs
+            uint64_t acch[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
             for (int c2 = 0; c2 < kBlockN / 2; ++c2) {
-                const float p0 = ptx::ex2_approx(fmaf(__uint_as_float(s[2 * c2]), cl, -msub));
-                const float p1 = ptx::ex2_approx(fmaf(__uint_as_float(s[2 * c2 + 1]), cl, -msub));
+                const uint64_t x = ptx::f32x2(__uint_as_float(s[2 * c2]), __uint_as_float(s[2 * c2 + 1]));
+                float y0, y1;
+                ptx::f32x2_split(ptx::fma_f32x2(x, cc2, nm2), y0, y1);
+                const float p0 = ptx::ex2_approx(y0);
+                const float p1 = ptx::ex2_approx(y1);
                 const uint32_t pk = ptx::pack_bf16x2(p0, p1);
-                sum[c2 & 3] += p0 + p1;
-                sumh[c2 & 3] += ptx::bf16lo_to_f32(pk) + ptx::bf16hi_to_f32(pk);
+                acc[c2 & 3] = ptx::add_f32x2(acc[c2 & 3], ptx::f32x2(p0, p1));
+                acch[c2 & 3] = ptx::add_f32x2(acch[c2 & 3], ptx::f32x2(ptx::bf16lo_to_f32(pk), ptx::bf16hi_to_f32(pk)));
                 s[c2] = pk;
             }
-            l = l * alpha + ((sum[0] + sum[1]) + (sum[2] + sum[3]));
-            lh = lh * alpha + ((sumh[0] + sumh[1]) + (sumh[2] + sumh[3]));
+            float sum = 0.f, sumh = 0.f;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                float a0, a1, h0, h1;
+                ptx::f32x2_split(acc[t], a0, a1);
+                ptx::f32x2_split(acch[t], h0, h1);
+                sum += a0 + a1;
+                sumh += h0 + h1;
+            }
+            l = l * alpha + sum;
+            lh = lh * alpha + sumh;
             ptx::tmem_st32(tS + 0, s);
             ptx::tmem_st32(tS + 32, s + 32);
             ptx::tmem_wait_st();
@@ -477,13 +511,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ubeg = p.cta_off[blockIdx.x];
     const int uend = p.cta_off[blockIdx.x + 1];
 
-    if (warp == kWarpProducer) {
-        if (lane == 0) run_producer<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, abort_flag);
-        __syncwarp();
-    } else if (warp == kWarpMma) {
-        if (lane == 0) run_mma<D>(p, ubeg, uend, tmem, sQ, sRing, sBar, abort_flag);
-        __syncwarp();
-    } else if (warp >= kWarpSoftmax) {
+    // Each register-budget change dominates only its own role's code, so the
+    // compiler can allocate the softmax path with the larger budget.
+    if (warp < kWarpSoftmax) {
+        ptx::setmaxnreg_dec<kRegsControl>();
+        if (warp == kWarpProducer) {
+            if (lane == 0) run_producer<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, abort_flag);
+            __syncwarp();
+        } else if (warp == kWarpMma) {
+            if (lane == 0) run_mma<D>(p, ubeg, uend, tmem, sQ, sRing, sBar, abort_flag);
+            __syncwarp();
+        }
+    } else {
+        ptx::setmaxnreg_inc<kRegsSoftmax>();
         run_softmax<D>(p, ubeg, uend, tmem, sBar, warp, lane, abort_flag);
     }
 
@@ -558,6 +598,17 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
             if (e != cudaSuccess) return e;
             if (dev >= 0 && dev < 128) attr_done[dev] = true;
         }
+    }
+    {
+        // The warpgroup register split assumes exactly kLaunchRegs registers
+        // per thread at launch; never launch a build that differs.
+        static std::once_flag once;
+        static int regs = -1;
+        std::call_once(once, [] {
+            cudaFuncAttributes fa;
+            if (cudaFuncGetAttributes(&fa, opattn_prefill_kernel<D>) == cudaSuccess) regs = fa.numRegs;
+        });
+        if (regs != kLaunchRegs) return -6;
     }
     KParams kp;
     kp.units = a.units;
