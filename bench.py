@@ -123,7 +123,7 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         for line in out.strip().splitlines():
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 9:
@@ -133,13 +133,21 @@ class ClockSampler:
                 mx.append(float(parts[2]))
             except ValueError:
                 continue
+            try:
+                pw.append(float(parts[3]))
+            except ValueError:
+                pass
             for name, val in zip(self.NAMES, parts[5:9]):
                 if val.lower() == "active":
                     reasons.add(name)
         if not sm:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm), "sm_mhz_min": min(sm)}
+        res = {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+               "samples": len(sm), "sm_mhz_min": min(sm)}
+        if pw:
+            res["power_w_median"] = statistics.median(pw)
+            res["power_w_max"] = max(pw)
+        return res
 
 
 def gpu_selector(torch, dev):

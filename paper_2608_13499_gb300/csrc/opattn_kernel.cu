@@ -47,10 +47,9 @@ constexpr int kWarpSoftmax = 4;  // first softmax warp; warps 4..7 -> M-tile 0, 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: no legitimate wait comes close
 constexpr uint64_t kForcedLimitNs = 20000000ull;  // 20 ms: the forced-timeout test
 constexpr uint64_t kDrainLimitNs = 200000000ull;  // in-flight copies / MMAs after an abort
-// Rescale O only when a row's running maximum grows by more than 2^8: the
-// final division by l uses the same stale maximum, so the result is exact;
-// probabilities stay below 2^8, far inside bf16 and fp32 range.
-constexpr float kRescaleThreshold = 8.0f;
+// Largest sum of one tile's exponentials accepted with a reused subtraction
+// base; fp32 sums and the fp32 O accumulator stay far from overflow.
+constexpr float kMaxTileSum = 18446744073709551616.0f;  // 2^64
 constexpr float kLn2 = 0.693147180559945309f;
 // Register split: the kernel is compiled for 168 registers per thread at
 // launch (384 threads, one CTA per SM = 64512 registers).  Warpgroup 0
@@ -299,6 +298,70 @@ __device__ __forceinline__ void run_mma(const KParams& p, int ubeg, int uend, ui
     drain_wait(bar(C::kBarDrain), 0u, kDrainLimitNs);
 }
 
+// N consecutive TMEM columns of this thread's lane into registers.
+template <int N>
+__device__ __forceinline__ void load_row(uint32_t taddr, uint32_t* r) {
+#pragma unroll
+    for (int c = 0; c < N; c += 32) ptx::tmem_ld32(taddr + c, r + c);
+    ptx::tmem_wait_ld();
+    ptx::tmem_ld_fence<N>(r);
+}
+
+// Scores of keys beyond this row's last visible key (column > last) -> -inf.
+__device__ __forceinline__ void mask_row(uint32_t* s, int last) {
+#pragma unroll
+    for (int c = 0; c < kBlockN; ++c)
+        if (c > last) s[c] = __float_as_uint(-INFINITY);
+}
+
+// Row max of 128 scores: 8 independent chains of 16, 3-input max.
+__device__ __forceinline__ float row_max(const uint32_t* s) {
+    float mx[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+        const uint32_t* v = s + 16 * t;
+        float a = ptx::max3f(__uint_as_float(v[0]), __uint_as_float(v[1]), __uint_as_float(v[2]));
+#pragma unroll
+        for (int i = 3; i < 15; i += 2) a = ptx::max3f(a, __uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+        mx[t] = fmaxf(a, __uint_as_float(v[15]));
+    }
+    return ptx::max3f(ptx::max3f(mx[0], mx[1], mx[2]), ptx::max3f(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7]));
+}
+
+// p = 2^(s*c - m) for the 128 scores of this row, packed in place as bf16
+// pairs into s[0..63]; `sum` gets the sum of the fp32 values, `sumh` the
+// sum of the bf16-rounded values the PV MMA consumes.  Per pair: one packed
+// FMA, two ex2, one bf16x2 pack, one packed add and two mixed-precision adds.
+__device__ __forceinline__ void exp_row(uint32_t* s, float c, float m, float& sum, float& sumh) {
+    const float msub = m == -INFINITY ? 0.f : m;
+    const uint64_t cc2 = ptx::f32x2(c, c);
+    const uint64_t nm2 = ptx::f32x2(-msub, -msub);
+    uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};  // (0.f, 0.f) pairs
+    float hs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int c2 = 0; c2 < kBlockN / 2; ++c2) {
+        const uint64_t x = ptx::f32x2(__uint_as_float(s[2 * c2]), __uint_as_float(s[2 * c2 + 1]));
+        float y0, y1;
+        ptx::f32x2_split(ptx::fma_f32x2(x, cc2, nm2), y0, y1);
+        const float p0 = ptx::ex2_approx(y0);
+        const float p1 = ptx::ex2_approx(y1);
+        const uint32_t pk = ptx::pack_bf16x2(p0, p1);
+        acc[c2 & 3] = ptx::add_f32x2(acc[c2 & 3], ptx::f32x2(p0, p1));
+        hs[(c2 & 3) * 2] = ptx::add_bf16lo(hs[(c2 & 3) * 2], pk);
+        hs[(c2 & 3) * 2 + 1] = ptx::add_bf16hi(hs[(c2 & 3) * 2 + 1], pk);
+        s[c2] = pk;
+    }
+    float a = 0.f;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+        float a0, a1;
+        ptx::f32x2_split(acc[t], a0, a1);
+        a += a0 + a1;
+    }
+    sum = a;
+    sumh = ((hs[0] + hs[1]) + (hs[2] + hs[3])) + ((hs[4] + hs[5]) + (hs[6] + hs[7]));
+}
+
 template <int D>
 __device__ __forceinline__ void store_zero_row(const KParams& p, int64_t row_idx) {
     uint4* dst = reinterpret_cast<uint4*>(p.o + row_idx * D);
@@ -336,7 +399,7 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
         }
         const int lim = min(u.qlim0 + tok, u.Lk - 1);                 // this row's last visible key
         const int tile_min_lim = min(u.qlim0 + mt * TPB, u.Lk - 1);  // smallest limit in the M-tile
-        float m = -INFINITY;  // running max, log2 domain
+        float m = -INFINITY;  // subtraction base, log2 domain
         float l = 0.f;        // running sum of the probabilities (fp32, for LSE)
         float lh = 0.f;       // running sum of the bf16-rounded probabilities PV consumes (normalises O)
         for (int j = 0; j < u.n_tiles; ++j) {
@@ -345,69 +408,39 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
             s_par ^= 1u;
             ptx::tc_fence_after();
             uint32_t s[kBlockN];
-            ptx::tmem_ld32(tS + 0, s);
-            ptx::tmem_ld32(tS + 32, s + 32);
-            ptx::tmem_ld32(tS + 64, s + 64);
-            ptx::tmem_ld32(tS + 96, s + 96);
-            ptx::tmem_wait_ld();
-            ptx::tmem_ld_fence<kBlockN>(s);
-
+            load_row<kBlockN>(tS, s);
             const int kbase = j * kBlockN;
-            if (kbase + kBlockN - 1 > tile_min_lim) {  // diagonal or tail tile: mask per row
-                const int lloc = lim - kbase;
-#pragma unroll
-                for (int c = 0; c < kBlockN; ++c)
-                    if (c > lloc) s[c] = __float_as_uint(-INFINITY);
-            }
-            // row max: 8 independent chains of 16 scores, 3-input max
-            float mx[8];
-#pragma unroll
-            for (int t = 0; t < 8; ++t) {
-                const uint32_t* v = s + 16 * t;
-                float a = ptx::max3f(__uint_as_float(v[0]), __uint_as_float(v[1]), __uint_as_float(v[2]));
-#pragma unroll
-                for (int i = 3; i < 15; i += 2) a = ptx::max3f(a, __uint_as_float(v[i]), __uint_as_float(v[i + 1]));
-                mx[t] = fmaxf(a, __uint_as_float(v[15]));
-            }
-            const float mraw = ptx::max3f(ptx::max3f(mx[0], mx[1], mx[2]), ptx::max3f(mx[3], mx[4], mx[5]),
-                                          fmaxf(mx[6], mx[7]));
-            const float m_tile = mraw * cl;
+            const bool masked = kbase + kBlockN - 1 > tile_min_lim;  // diagonal or tail tile
+            if (masked) mask_row(s, lim - kbase);
+            // Subtraction base m: the exact row max on the unit's first tile
+            // (and while some row of the warp has none yet); later tiles reuse
+            // it, since O / l and LSE = m + log2(l) are exact for any base.
+            // A tile whose exponentials sum beyond kMaxTileSum is redone with
+            // its own exact max (O and the sums rescaled).
             float alpha = 1.f;
             bool rescale = false;
-            if (j == 0) {
-                m = m_tile;
-            } else if (m_tile > m + kRescaleThreshold) {
-                alpha = ptx::ex2_approx(m - m_tile);
-                m = m_tile;
-                rescale = true;
+            if (__any_sync(0xFFFFFFFFu, j == 0 || m == -INFINITY)) {
+                const float m_tile = row_max(s) * cl;
+                if (j == 0) {
+                    m = m_tile;
+                } else if (m_tile > m) {
+                    alpha = m == -INFINITY ? 0.f : ptx::ex2_approx(m - m_tile);
+                    m = m_tile;
+                    rescale = true;
+                }
             }
-            const float msub = (m == -INFINITY) ? 0.f : m;
-            // p = 2^(s*c - m) on pairs: one packed FMA, two ex2, one bf16x2
-            // pack, two packed adds (exact and rounded running sums)
-            const uint64_t cc2 = ptx::f32x2(cl, cl);
-            const uint64_t nm2 = ptx::f32x2(-msub, -msub);
-            uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};   // (0.f, 0.f) pairs
-            uint64_t acch[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-            for (int c2 = 0; c2 < kBlockN / 2; ++c2) {
-                const uint64_t x = ptx::f32x2(__uint_as_float(s[2 * c2]), __uint_as_float(s[2 * c2 + 1]));
-                float y0, y1;
-                ptx::f32x2_split(ptx::fma_f32x2(x, cc2, nm2), y0, y1);
-                const float p0 = ptx::ex2_approx(y0);
-                const float p1 = ptx::ex2_approx(y1);
-                const uint32_t pk = ptx::pack_bf16x2(p0, p1);
-                acc[c2 & 3] = ptx::add_f32x2(acc[c2 & 3], ptx::f32x2(p0, p1));
-                acch[c2 & 3] = ptx::add_f32x2(acch[c2 & 3], ptx::f32x2(ptx::bf16lo_to_f32(pk), ptx::bf16hi_to_f32(pk)));
-                s[c2] = pk;
-            }
-            float sum = 0.f, sumh = 0.f;
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-                float a0, a1, h0, h1;
-                ptx::f32x2_split(acc[t], a0, a1);
-                ptx::f32x2_split(acch[t], h0, h1);
-                sum += a0 + a1;
-                sumh += h0 + h1;
+            float sum, sumh;
+            exp_row(s, cl, m, sum, sumh);
+            if (__any_sync(0xFFFFFFFFu, !(sum <= kMaxTileSum))) {
+                load_row<kBlockN>(tS, s);
+                if (masked) mask_row(s, lim - kbase);
+                const float m_tile = row_max(s) * cl;
+                if (m_tile > m) {
+                    alpha *= m == -INFINITY ? 0.f : ptx::ex2_approx(m - m_tile);
+                    m = m_tile;
+                    rescale = true;
+                }
+                exp_row(s, cl, m, sum, sumh);
             }
             l = l * alpha + sum;
             lh = lh * alpha + sumh;
@@ -418,9 +451,7 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
 #pragma unroll
                 for (int ch = 0; ch < D / 32; ++ch) {
                     uint32_t ov[32];
-                    ptx::tmem_ld32(tO + 32 * ch, ov);
-                    ptx::tmem_wait_ld();
-                    ptx::tmem_ld_fence<32>(ov);
+                    load_row<32>(tO + 32 * ch, ov);
 #pragma unroll
                     for (int t = 0; t < 32; ++t) ov[t] = __float_as_uint(__uint_as_float(ov[t]) * alpha);
                     ptx::tmem_st32(tO + 32 * ch, ov);

@@ -232,6 +232,21 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
 }
+// acc + (bf16 in bits 0-15 / 16-31 of `packed`), one mixed-precision add.
+__device__ __forceinline__ float add_bf16lo(float acc, uint32_t packed) {
+    float r;
+    asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.bf16 %0, lo, %2;\n\t}"
+        : "=f"(r)
+        : "r"(packed), "f"(acc));
+    return r;
+}
+__device__ __forceinline__ float add_bf16hi(float acc, uint32_t packed) {
+    float r;
+    asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.bf16 %0, hi, %2;\n\t}"
+        : "=f"(r)
+        : "r"(packed), "f"(acc));
+    return r;
+}
 __device__ __forceinline__ float bf16lo_to_f32(uint32_t packed) { return __uint_as_float(packed << 16); }
 __device__ __forceinline__ float bf16hi_to_f32(uint32_t packed) {
     return __uint_as_float(packed & 0xFFFF0000u);

@@ -90,6 +90,24 @@ def test_large_logits_exercise_rescaling():
     check(o, lse, o_ref, lse_ref, w.name)
 
 
+def test_growing_logits_force_tiles_to_be_redone():
+    """Logits grow by ~0.09 nats per key along each prompt (up to ~96 nats), so
+    a tile's exponentials over the subtraction base of an earlier tile pass the
+    kernel's overflow guard and tiles are recomputed with their own maximum."""
+    w = custom("growing", [1024, 300], [1024, 300], 8, 2, 64, seed=9)
+    q, k, v = W.make_inputs(w, "cuda")
+    pos = torch.cat([torch.arange(n, dtype=torch.float32) for n in w.k_lens]).to("cuda")
+    qf = q.float() * 0.1
+    qf[:, :, 0] = 24.0
+    kf = k.float() * 0.1
+    kf[:, :, 0] = (pos / 32.0)[:, None]
+    q, k = qf.to(torch.bfloat16), kf.to(torch.bfloat16)
+    o, lse = run_gpu(w, q, k, v)
+    o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
+    assert lse_ref.max() > 60.0  # the logits really span far beyond one tile's range
+    check(o, lse, o_ref, lse_ref, w.name)
+
+
 def sample_rows(w, rng, n_random):
     tok, hd = [], []
     G = w.Hq // w.Hkv
