@@ -11,7 +11,7 @@
 //
 // CTA layout (384 threads, one CTA per SM, persistent over its unit list):
 //   warp 0        TMA producer: Q tiles of the unit, then K_j, V_j into a ring
-//   warp 1        TMEM owner + single-thread MMA issuer
+//   warp 1        TMEM owner + MMA issuer (whole warp, one elected lane issues)
 //   warps 2-3     idle
 //   warps 4-7     softmax / correction / epilogue of M-tile 0 (one row per thread)
 //   warps 8-11    the same for M-tile 1
@@ -205,8 +205,8 @@ __device__ __forceinline__ void issue_s(uint32_t tmem, int mt, uint32_t sQ, uint
     for (int ks = 0; ks < D / 16; ++ks) {
         const uint32_t qoff = (ks >> 2) * (kRowsPerTile * 128) + (ks & 3) * 32;
         const uint32_t koff = (ks >> 2) * (kBlockN * 128) + (ks & 3) * 32;
-        ptx::mma_ss(d_tmem, ptx::sdesc_sw128(qbase + qoff, 16, 1024), ptx::sdesc_sw128(sK + koff, 16, 1024),
-                    C::kIdescS, ks > 0 ? 1u : 0u);
+        ptx::mma_ss_warp(d_tmem, ptx::sdesc_sw128(qbase + qoff, 16, 1024), ptx::sdesc_sw128(sK + koff, 16, 1024),
+                         C::kIdescS, ks > 0 ? 1u : 0u);
     }
 }
 
@@ -219,8 +219,8 @@ __device__ __forceinline__ void issue_pv(uint32_t tmem, int mt, uint32_t sV, boo
     for (int ks = 0; ks < kBlockN / 16; ++ks) {
         // V tile is [keys][d] (MN-major for this product): 16 keys per step,
         // 64-column blocks kBlockN * 128 bytes apart, 8-key groups 1024 apart.
-        ptx::mma_ts(d_tmem, a_tmem + ks * 8, ptx::sdesc_sw128(sV + ks * (16 * 128), kBlockN * 128, 1024),
-                    C::kIdescPV, (accumulate || ks > 0) ? 1u : 0u);
+        ptx::mma_ts_warp(d_tmem, a_tmem + ks * 8, ptx::sdesc_sw128(sV + ks * (16 * 128), kBlockN * 128, 1024),
+                         C::kIdescPV, (accumulate || ks > 0) ? 1u : 0u);
     }
 }
 
@@ -232,69 +232,75 @@ __device__ __forceinline__ void run_mma(const KParams& p, int ubeg, int uend, ui
     auto slot_addr = [&](uint32_t s) { return sRing + s * C::kSlotBytes; };
     uint32_t slot = 0, ring_par = 0, q_uses = 0;
     uint32_t p_par[2] = {0u, 0u};
+    // Run by all 32 lanes of the MMA warp: waits are made warp-uniform and one
+    // elected lane issues each MMA and commit.
+    auto wait = [&](int b, uint32_t parity) {
+        return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
+    };
     bool ok = true;
-    if (p.flags & kFlagForceTimeout) ok = bounded_wait(bar(C::kBarNever), 0u, abort_flag, p.status, kForcedLimitNs);
+    if (p.flags & kFlagForceTimeout)
+        ok = __all_sync(0xFFFFFFFFu, bounded_wait(bar(C::kBarNever), 0u, abort_flag, p.status, kForcedLimitNs));
 
     for (int ui = ubeg; ui < uend && ok; ++ui) {
         const UnitRec u = p.units[ui];
         const int nT = u.n_tiles;
         if (nT <= 0) continue;
         // prologue: S0(0), S1(0)
-        if (!(ok = bounded_wait(bar(C::kBarQFull + 0), q_uses & 1u, abort_flag, p.status, kWaitLimitNs))) break;
+        if (!(ok = wait(C::kBarQFull + 0, q_uses & 1u))) break;
         uint32_t kslot = slot;
-        if (!(ok = bounded_wait(bar(C::kBarFull + kslot), ring_par, abort_flag, p.status, kWaitLimitNs))) break;
+        if (!(ok = wait(C::kBarFull + kslot, ring_par))) break;
         if (++slot == C::kSlots) { slot = 0; ring_par ^= 1u; }
         ptx::tc_fence_after();
         issue_s<D>(tmem, 0, sQ, slot_addr(kslot));
-        ptx::tc_commit(bar(C::kBarS + 0));
-        if (nT == 1) ptx::tc_commit(bar(C::kBarQEmpty + 0));
-        if (!(ok = bounded_wait(bar(C::kBarQFull + 1), q_uses & 1u, abort_flag, p.status, kWaitLimitNs))) break;
+        ptx::tc_commit_warp(bar(C::kBarS + 0));
+        if (nT == 1) ptx::tc_commit_warp(bar(C::kBarQEmpty + 0));
+        if (!(ok = wait(C::kBarQFull + 1, q_uses & 1u))) break;
         ptx::tc_fence_after();
         issue_s<D>(tmem, 1, sQ, slot_addr(kslot));
-        ptx::tc_commit(bar(C::kBarS + 1));
-        if (nT == 1) ptx::tc_commit(bar(C::kBarQEmpty + 1));
-        ptx::tc_commit(bar(C::kBarEmpty + kslot));
+        ptx::tc_commit_warp(bar(C::kBarS + 1));
+        if (nT == 1) ptx::tc_commit_warp(bar(C::kBarQEmpty + 1));
+        ptx::tc_commit_warp(bar(C::kBarEmpty + kslot));
         ++q_uses;
 
         for (int j = 0; j < nT; ++j) {
             const uint32_t vslot = slot;
-            if (!(ok = bounded_wait(bar(C::kBarFull + vslot), ring_par, abort_flag, p.status, kWaitLimitNs))) break;
+            if (!(ok = wait(C::kBarFull + vslot, ring_par))) break;
             if (++slot == C::kSlots) { slot = 0; ring_par ^= 1u; }
             const bool more = j + 1 < nT;
             // M-tile 0
-            if (!(ok = bounded_wait(bar(C::kBarP + 0), p_par[0], abort_flag, p.status, kWaitLimitNs))) break;
+            if (!(ok = wait(C::kBarP + 0, p_par[0]))) break;
             p_par[0] ^= 1u;
             ptx::tc_fence_after();
             issue_pv<D>(tmem, 0, slot_addr(vslot), j > 0);
             if (more) {
                 kslot = slot;
-                if (!(ok = bounded_wait(bar(C::kBarFull + kslot), ring_par, abort_flag, p.status, kWaitLimitNs)))
+                if (!(ok = wait(C::kBarFull + kslot, ring_par)))
                     break;
                 if (++slot == C::kSlots) { slot = 0; ring_par ^= 1u; }
                 issue_s<D>(tmem, 0, sQ, slot_addr(kslot));
-                if (j + 2 == nT) ptx::tc_commit(bar(C::kBarQEmpty + 0));
-                ptx::tc_commit(bar(C::kBarS + 0));
+                if (j + 2 == nT) ptx::tc_commit_warp(bar(C::kBarQEmpty + 0));
+                ptx::tc_commit_warp(bar(C::kBarS + 0));
             } else {
-                ptx::tc_commit(bar(C::kBarO + 0));
+                ptx::tc_commit_warp(bar(C::kBarO + 0));
             }
             // M-tile 1
-            if (!(ok = bounded_wait(bar(C::kBarP + 1), p_par[1], abort_flag, p.status, kWaitLimitNs))) break;
+            if (!(ok = wait(C::kBarP + 1, p_par[1]))) break;
             p_par[1] ^= 1u;
             ptx::tc_fence_after();
             issue_pv<D>(tmem, 1, slot_addr(vslot), j > 0);
             if (more) {
                 issue_s<D>(tmem, 1, sQ, slot_addr(kslot));
-                if (j + 2 == nT) ptx::tc_commit(bar(C::kBarQEmpty + 1));
-                ptx::tc_commit(bar(C::kBarS + 1));
-                ptx::tc_commit(bar(C::kBarEmpty + kslot));
+                if (j + 2 == nT) ptx::tc_commit_warp(bar(C::kBarQEmpty + 1));
+                ptx::tc_commit_warp(bar(C::kBarS + 1));
+                ptx::tc_commit_warp(bar(C::kBarEmpty + kslot));
             } else {
-                ptx::tc_commit(bar(C::kBarO + 1));
+                ptx::tc_commit_warp(bar(C::kBarO + 1));
             }
-            ptx::tc_commit(bar(C::kBarEmpty + vslot));
+            ptx::tc_commit_warp(bar(C::kBarEmpty + vslot));
         }
     }
-    // Every MMA this thread issued must finish before TMEM is released.
-    ptx::tc_commit(bar(C::kBarDrain));
+    // Every MMA this warp issued must finish before TMEM is released.
+    ptx::tc_commit_warp(bar(C::kBarDrain));
     drain_wait(bar(C::kBarDrain), 0u, kDrainLimitNs);
 }
 
@@ -550,8 +556,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) run_producer<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, abort_flag);
             __syncwarp();
         } else if (warp == kWarpMma) {
-            if (lane == 0) run_mma<D>(p, ubeg, uend, tmem, sQ, sRing, sBar, abort_flag);
-            __syncwarp();
+            run_mma<D>(p, ubeg, uend, tmem, sQ, sRing, sBar, abort_flag);
         }
     } else {
         ptx::setmaxnreg_inc<kRegsSoftmax>();
