@@ -339,14 +339,7 @@ def run_ours(args, w):
     if rank == 0:
         peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
         peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-        traffic = None
-        tpath = os.path.join(ROOT, "profiles", "traffic.json")
-        if os.path.exists(tpath):
-            with open(tpath) as f:
-                tj = json.load(f)
-            entry = tj.get(w.name)
-            if entry and entry.get("kernel_rev") == kernel_revision():
-                traffic = entry.get("bytes_per_launch")
+        traffic = recorded_traffic(w.name)
         line = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": elapsed_max / args.steps * 1e3, "higher_is_better": True,
@@ -373,6 +366,21 @@ def run_ours(args, w):
         dist.barrier()
         dist.destroy_process_group()
     return 0
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch from the committed ncu record, or None when the
+    kernel sources changed since that capture (the counters no longer apply)."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    rev = kernel_revision()
+    with open(path) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) == 3 and not line.startswith("#") and parts[0] == workload and parts[1] == rev:
+                return int(parts[2])
+    return None
 
 
 def kernel_revision() -> str:
