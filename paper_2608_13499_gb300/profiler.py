@@ -1,0 +1,374 @@
+"""Operator profile of the prefill-attention operator.
+
+OpScale provisions each operator from a profile of its latency over batch
+size B, prompt length L and SM share S (§4.1, "Operator Profiling Space"),
+built by sparse sampling: random points of the (B, L) space are measured and
+unsampled points are estimated by non-parametric piecewise interpolation
+(§4.2).  Operators that are structurally identical (the same attention in
+every layer, or in two models with the same head geometry) share one profile
+(§4.2, structural equivalence).  This module does that for libopattn:
+
+* ``PiecewiseProfile``: piecewise-linear interpolation of log T over the log
+  of each coordinate ((B, L) or (B, L, S)) on a Delaunay triangulation of the
+  sampled points.  In log space the operator's O(L^2 B) cost (§2.1) is close
+  to linear, so few samples suffice.  The corners of the sampled box are
+  always in the sample, so every query inside the box is inside the
+  triangulation.
+* ``sample_points``: random points (a Latin hypercube in log space) plus
+  the box corners.
+* ``ProfileStore``: profiles keyed by the operator's structure, so that each
+  distinct attention shape of a model is measured once.
+* ``measure_ms``: CUDA-event time of one launch (``opattn_plan_run``) for a
+  batch of B prompts of L tokens, with the persistent grid optionally capped
+  at ``max_ctas`` CTAs.  The kernel keeps one CTA per SM, so the cap is the
+  operator's SM budget S (the paper's S_v, §3.1).
+* ``sm_budget_curve``: latency against SM share for a workload.
+* ``profile_accuracy``: relative error of an interpolated profile on
+  held-out random points.  The paper's operator profiles reach 7% mean and
+  15% P90 relative error (§5, "Profiling-driven Model Accuracy").
+
+``python -m paper_2608_13499_gb300.profiler --out FILE`` on a GPU writes a
+markdown report of the studies.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import statistics
+from dataclasses import asdict, dataclass
+
+import numpy as np
+
+
+class PiecewiseProfile:
+    """Piecewise-linear interpolation of log T over log-coordinates.
+
+    ``coords`` is an (n, k) array of positive sample coordinates (k = 2 for
+    (B, L), 3 for (B, L, S)), ``times_ms`` the n measured latencies.
+    """
+
+    def __init__(self, coords, times_ms):
+        from scipy.interpolate import LinearNDInterpolator
+        x = np.asarray(coords, dtype=np.float64)
+        t = np.asarray(times_ms, dtype=np.float64)
+        if x.ndim != 2 or len(x) != len(t):
+            raise ValueError("coords must be (n, k) with one time per row")
+        if len(t) < x.shape[1] + 1:
+            raise ValueError(f"need at least {x.shape[1] + 1} samples in {x.shape[1]} dimensions")
+        if np.any(x <= 0) or np.any(t <= 0) or not np.all(np.isfinite(t)):
+            raise ValueError("coordinates and times must be positive")
+        self.coords = x
+        self.times_ms = t
+        self._x = np.log(x)
+        self._logt = np.log(t)
+        self._interp = LinearNDInterpolator(self._x, self._logt)
+
+    @property
+    def dims(self) -> int:
+        return self.coords.shape[1]
+
+    def predict(self, coords) -> np.ndarray:
+        """Estimated times (ms) at an (m, k) array of points.
+
+        Outside the convex hull of the samples the nearest sample (in log
+        coordinates) answers, so the profile never extrapolates.
+        """
+        x = np.log(np.atleast_2d(np.asarray(coords, dtype=np.float64)))
+        if x.shape[1] != self.dims:
+            raise ValueError(f"points have {x.shape[1]} coordinates, the profile {self.dims}")
+        out = np.asarray(self._interp(x), dtype=np.float64).reshape(len(x))
+        miss = ~np.isfinite(out)
+        if miss.any():
+            d = ((x[miss, None, :] - self._x[None, :, :]) ** 2).sum(-1)
+            out[miss] = self._logt[d.argmin(axis=1)]
+        return np.exp(out)
+
+    def to_dict(self) -> dict:
+        return {"coords": self.coords.tolist(), "times_ms": self.times_ms.tolist()}
+
+    @classmethod
+    def from_dict(cls, d: dict) -> "PiecewiseProfile":
+        return cls(d["coords"], d["times_ms"])
+
+
+def sample_points(n: int, rng, ranges, integer=None, corners: bool = True, stratified: bool = True) -> np.ndarray:
+    """(n [+ 2^k], k) random points, log-uniform in each range of ``ranges``.
+
+    ``stratified`` draws a Latin hypercube in log space (each coordinate's
+    log range cut into n equal strata, one point per stratum, strata paired
+    at random across coordinates), which avoids the long thin triangles that
+    clustered plain random points leave.  ``integer[i]`` rounds coordinate i
+    (batch size, length); ``corners`` prepends the 2^k corners of the box.
+    """
+    k = len(ranges)
+    integer = [True] * k if integer is None else list(integer)
+    cols = []
+    for (lo, hi), is_int in zip(ranges, integer):
+        u = (rng.permutation(n) + rng.uniform(0.0, 1.0, n)) / n if stratified else rng.uniform(0.0, 1.0, n)
+        c = np.exp(math.log(lo) + u * (math.log(hi) - math.log(lo)))
+        if is_int:
+            c = np.rint(c)
+        cols.append(np.clip(c, lo, hi))
+    pts = np.column_stack(cols) if n else np.zeros((0, k))
+    if corners:
+        box = np.array([[ranges[i][(m >> i) & 1] for i in range(k)] for m in range(1 << k)], dtype=np.float64)
+        pts = np.concatenate([box, pts])
+    return pts
+
+
+def relative_errors(predicted, measured) -> dict:
+    p, m = np.asarray(predicted, dtype=np.float64), np.asarray(measured, dtype=np.float64)
+    e = np.abs(p - m) / m
+    return {"mean": float(e.mean()), "p90": float(np.percentile(e, 90)), "max": float(e.max()), "n": int(len(e))}
+
+
+# ------------------------------------------------------- structural equivalence
+
+@dataclass(frozen=True)
+class OperatorKey:
+    """What decides an attention operator's latency: its kernel and head geometry.
+
+    Layers (and models) whose attention has the same key run the same kernel
+    on the same shapes, so one profile serves them all.
+    """
+    op: str
+    Hq: int
+    Hkv: int
+    d: int
+    dtype: str = "bf16"
+
+    def name(self) -> str:
+        return f"{self.op}/Hq{self.Hq}/Hkv{self.Hkv}/d{self.d}/{self.dtype}"
+
+
+def attention_key(Hq: int, Hkv: int, d: int) -> OperatorKey:
+    return OperatorKey("opattn_prefill", int(Hq), int(Hkv), int(d))
+
+
+class ProfileStore:
+    """Profiles by operator key; ``get`` profiles a key only the first time."""
+
+    def __init__(self):
+        self._profiles: dict = {}
+        self.measured: list = []     # keys in the order they were profiled
+
+    def __contains__(self, key: OperatorKey) -> bool:
+        return key in self._profiles
+
+    def __len__(self) -> int:
+        return len(self._profiles)
+
+    def get(self, key: OperatorKey, profile_fn) -> PiecewiseProfile:
+        if key not in self._profiles:
+            self._profiles[key] = profile_fn(key)
+            self.measured.append(key)
+        return self._profiles[key]
+
+    def profiles_for(self, layer_keys, profile_fn) -> list:
+        """One profile per layer, measuring each distinct key once."""
+        return [self.get(k, profile_fn) for k in layer_keys]
+
+    def save(self, path: str) -> None:
+        blob = [{"key": asdict(k), "profile": p.to_dict()} for k, p in self._profiles.items()]
+        with open(path, "w") as f:
+            json.dump(blob, f)
+
+    @classmethod
+    def load(cls, path: str) -> "ProfileStore":
+        s = cls()
+        with open(path) as f:
+            for e in json.load(f):
+                s._profiles[OperatorKey(**e["key"])] = PiecewiseProfile.from_dict(e["profile"])
+        return s
+
+
+# ---------------------------------------------------------------- GPU side
+
+class _Buffers:
+    """Device inputs sized for the largest point; every point uses a prefix."""
+
+    def __init__(self, max_tokens: int, Hq: int, Hkv: int, d: int, device="cuda"):
+        import torch
+
+        from . import workloads as W
+        self.Hq, self.Hkv, self.d = Hq, Hkv, d
+        n = max_tokens
+        self.q = W.normal_bf16(0, W.STREAM_Q, n * Hq * d, device).view(n, Hq, d)
+        self.k = W.normal_bf16(0, W.STREAM_K, n * Hkv * d, device).view(n, Hkv, d)
+        self.v = W.normal_bf16(0, W.STREAM_V, n * Hkv * d, device).view(n, Hkv, d)
+        self.o = torch.empty((n, Hq, d), dtype=torch.bfloat16, device=device)
+        self.lse = torch.empty((n, Hq), dtype=torch.float32, device=device)
+
+
+def _time_plan_ms(plan, q, k, v, o, lse, scale, reps: int, warm_ms: float = 25.0, min_ms: float = 2.0) -> float:
+    """Median per-launch CUDA-event time (ms) of ``plan.run`` on the current stream.
+
+    The operator first runs back to back for ``warm_ms`` so the clocks leave
+    their idle state.  Each of the ``reps`` samples then times ``inner``
+    back-to-back launches between two events (``inner`` chosen so a sample
+    spans at least ``min_ms``), so the host's launch gap before a single short
+    launch is not counted.
+    """
+    import torch
+    stream = torch.cuda.current_stream()
+
+    def sample(inner):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(inner):
+            plan.run(q, k, v, o, lse, scale, stream)
+        b.record(stream)
+        b.synchronize()
+        return a.elapsed_time(b) / inner
+
+    first = sample(1)
+    inner = max(1, min(256, int(math.ceil(min_ms / max(first, 1e-3)))))
+    warm = 0.0
+    while warm < warm_ms:
+        warm += sample(inner) * inner
+    return statistics.median(sample(inner) for _ in range(reps))
+
+
+def n_sms() -> int:
+    import torch
+    return torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+
+
+def ctas_for_share(share: float, sms: int) -> int:
+    """SM count for an SM share in (0, 1]: round(share * sms), at least 1."""
+    return max(1, min(sms, int(round(share * sms))))
+
+
+def measure_ms(buf, B: int, L: int, max_ctas: int = 0, reps: int = 5) -> float:
+    """Median time (ms) of one launch for B prompts of L tokens each (q_len = kv_len = L)."""
+    import paper_2608_13499_gb300 as pkg
+    cu = np.arange(B + 1, dtype=np.int32) * np.int32(L)
+    with pkg.Plan(cu, cu, buf.Hq, buf.Hkv, buf.d, max_ctas=max_ctas) as plan:
+        return _time_plan_ms(plan, buf.q, buf.k, buf.v, buf.o, buf.lse, buf.d ** -0.5, reps)
+
+
+def sm_budget_curve(w, ctas, reps: int = 5, device="cuda"):
+    """[(n_ctas, ms)] for workload w with the persistent grid capped at each budget."""
+    import torch
+
+    import paper_2608_13499_gb300 as pkg
+
+    from . import workloads as W
+    q, k, v = W.make_inputs(w, device)
+    o = torch.empty((w.total_q, w.Hq, w.d), dtype=torch.bfloat16, device=device)
+    lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device=device)
+    out = []
+    for n in ctas:
+        with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, max_ctas=n) as plan:
+            out.append((plan.n_ctas, _time_plan_ms(plan, q, k, v, o, lse, w.scale, reps)))
+    return out
+
+
+def profile_accuracy(n_train: int, n_test: int, seed: int = 0, key: OperatorKey = attention_key(32, 8, 128),
+                     b_range=(1, 32), l_range=(128, 8192), s_range=None, reps: int = 5):
+    """Fit a profile on n_train random points plus the box corners; error on n_test others.
+
+    With ``s_range`` (SM shares, e.g. (1/16, 1)) the profile is over (B, L, S).
+    """
+    rng = np.random.default_rng(seed)
+    ranges = [b_range, l_range] + ([s_range] if s_range else [])
+    integer = [True, True] + ([False] if s_range else [])
+    train = sample_points(n_train, rng, ranges, integer)
+    test = sample_points(n_test, rng, ranges, integer, corners=False, stratified=False)
+    buf = _Buffers(int(b_range[1] * l_range[1]), key.Hq, key.Hkv, key.d)
+    sms = n_sms()
+
+    def run(p):
+        ctas = ctas_for_share(p[2], sms) if s_range else 0
+        return measure_ms(buf, int(p[0]), int(p[1]), ctas, reps)
+
+    t_train = np.array([run(p) for p in train])
+    t_test = np.array([run(p) for p in test])
+    t_again = np.array([run(p) for p in test])
+    prof = PiecewiseProfile(train, t_train)
+    pred = prof.predict(test)
+    return {"profile": prof, "test": test, "measured": t_test, "predicted": pred,
+            "errors": relative_errors(pred, t_test), "noise": relative_errors(t_again, t_test),
+            "remeasured": t_again}
+
+
+def _accuracy_section(title, acc, n_train, k) -> list:
+    e = acc["errors"]
+    lines = [f"## {title}", "",
+             f"{len(acc['profile'].coords)} sampled points ({1 << k} box corners + {n_train} random points, "
+             f"a Latin hypercube in log space), {e['n']} held-out log-uniform random points.", "",
+             "| relative error of the interpolated latency | value |", "|---|---|",
+             f"| mean | {100 * e['mean']:.1f}% |", f"| P90 | {100 * e['p90']:.1f}% |",
+             f"| max | {100 * e['max']:.1f}% |", "",
+             f"Measurement noise (the held-out points timed twice): {100 * acc['noise']['mean']:.1f}% mean, "
+             f"{100 * acc['noise']['p90']:.1f}% P90.", "",
+             "| " + " | ".join(["B", "L", "S"][:k]) + " | measured (ms) | predicted (ms) |",
+             "|" + "---|" * (k + 2)]
+    for p, t, q in list(zip(acc["test"], acc["measured"], acc["predicted"]))[:10]:
+        cells = [str(int(p[0])), str(int(p[1]))] + ([f"{p[2]:.3f}"] if k == 3 else [])
+        lines.append("| " + " | ".join(cells) + f" | {t:.4f} | {q:.4f} |")
+    return lines + [""]
+
+
+def _report(args) -> str:
+    import torch
+
+    from . import workloads as W
+    sms = n_sms()
+    lines = ["# Operator profile of opattn_prefill: sparse sampling, piecewise interpolation, SM budget", "",
+             f"Command: `python -m paper_2608_13499_gb300.profiler --train {args.train} --test {args.test} "
+             f"--train3 {args.train3} --test3 {args.test3} --seed {args.seed} --reps {args.reps} --out <file>"
+             f"{' --dump <file>' if args.dump else ''}` "
+             f"on one {torch.cuda.get_device_name(0)} ({sms} SMs).", "",
+             "Operator: Llama-3-8B attention heads (Hq 32, Hkv 8, d 128), B prompts of L tokens each, "
+             "B in [1, 32], L in [128, 8192], inputs N(0, 1) bf16.  Each point is the median of "
+             f"{args.reps} CUDA-event samples after 25 ms of back-to-back warm-up launches; a sample times "
+             "enough back-to-back launches to span 2 ms and divides.  The paper's operator profiles: "
+             "7% mean and 15% P90 relative error.", ""]
+    acc2 = profile_accuracy(args.train, args.test, args.seed, reps=args.reps)
+    lines += _accuracy_section("Profile over (B, L) at the full GPU", acc2, args.train, 2)
+    acc3 = profile_accuracy(args.train3, args.test3, args.seed + 1, s_range=(1.0 / 16, 1.0), reps=args.reps)
+    lines += _accuracy_section("Profile over (B, L, S), SM share S in [1/16, 1]", acc3, args.train3, 3)
+    if args.dump:
+        blob = {name: {"train": a["profile"].to_dict(), "test": a["test"].tolist(),
+                       "measured": a["measured"].tolist(), "remeasured": a["remeasured"].tolist()}
+                for name, a in (("BL", acc2), ("BLS", acc3))}
+        with open(args.dump, "w") as f:
+            json.dump(blob, f)
+    shares = (0.125, 0.25, 0.5, 0.75, 1.0)
+    budgets = [ctas_for_share(f, sms) for f in shares]
+    lines += [f"## Latency against SM budget (persistent grid capped at n CTAs, one CTA per SM)", "",
+              "Time relative to the full GPU in parentheses; perfect scaling would be 1/share.", "",
+              "| workload | " + " | ".join(f"{b} SMs ({100 * b / sms:.0f}%)" for b in budgets) + " |",
+              "|---|" + "---|" * len(budgets)]
+    for name in ("llama3_8b", "llama3_70b", "bursty", "chunked"):
+        curve = sm_budget_curve(W.STANDARD[name](), budgets, reps=args.reps)
+        base = curve[-1][1]
+        lines.append(f"| {W.STANDARD[name]().name} | "
+                     + " | ".join(f"{ms:.3f} ms ({ms / base:.2f}x)" for _, ms in curve) + " |")
+    return "\n".join(lines) + "\n"
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description="profile opattn_prefill on the current GPU")
+    ap.add_argument("--train", type=int, default=80)
+    ap.add_argument("--test", type=int, default=40)
+    ap.add_argument("--train3", type=int, default=160)
+    ap.add_argument("--test3", type=int, default=40)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--reps", type=int, default=7)
+    ap.add_argument("--out", default=None)
+    ap.add_argument("--dump", default=None, help="write every measured point as JSON")
+    args = ap.parse_args(argv)
+    from . import build
+    build.build()
+    text = _report(args)
+    if args.out:
+        with open(args.out, "w") as f:
+            f.write(text)
+    print(text)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,42 @@
+"""Operator profile on the GPU: SM budget and sparse-sampling interpolation.
+
+Sanity bars only (the measured accuracy is reported by the profiler's own
+report): a smaller SM budget never makes the launch faster, an eighth of the
+SMs makes a compute-bound batch several times slower, and an interpolated
+profile from a handful of points predicts held-out points roughly.
+"""
+import numpy as np
+import pytest
+
+import paper_2608_13499_gb300 as pkg
+from paper_2608_13499_gb300 import build as pbuild
+from paper_2608_13499_gb300 import profiler as P
+from paper_2608_13499_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    pbuild.build()
+    return pkg.load()
+
+
+def test_latency_falls_with_sm_budget():
+    w = W.Workload("sm_budget_4x2048", [2048] * 4, [2048] * 4, 32, 8, 128)
+    sms = P.n_sms()
+    budgets = [P.ctas_for_share(f, sms) for f in (0.125, 0.25, 0.5, 1.0)]
+    curve = P.sm_budget_curve(w, budgets, reps=5)
+    assert [n for n, _ in curve] == budgets
+    ms = [t for _, t in curve]
+    for a, b in zip(ms, ms[1:]):
+        assert b <= a * 1.05, curve
+    assert ms[0] >= 4.0 * ms[-1], curve
+
+
+def test_small_profile_predicts_held_out_points():
+    acc = P.profile_accuracy(12, 8, seed=3, b_range=(1, 8), l_range=(128, 2048), reps=3)
+    assert np.all(acc["measured"] > 0)
+    assert acc["errors"]["mean"] < 0.25, acc["errors"]
+    prof = acc["profile"]
+    np.testing.assert_allclose(prof.predict(prof.coords), prof.times_ms, rtol=1e-9)
