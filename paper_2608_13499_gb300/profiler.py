@@ -127,23 +127,27 @@ def relative_errors(predicted, measured) -> dict:
 
 @dataclass(frozen=True)
 class OperatorKey:
-    """What decides an attention operator's latency: its kernel and head geometry.
+    """What decides an operator's latency: its kernel, shape parameters and dtype.
 
-    Layers (and models) whose attention has the same key run the same kernel
+    Layers (and models) whose operator has the same key run the same kernel
     on the same shapes, so one profile serves them all.
     """
     op: str
-    Hq: int
-    Hkv: int
-    d: int
+    shape: tuple
     dtype: str = "bf16"
 
     def name(self) -> str:
-        return f"{self.op}/Hq{self.Hq}/Hkv{self.Hkv}/d{self.d}/{self.dtype}"
+        return f"{self.op}{list(self.shape)}/{self.dtype}"
 
 
 def attention_key(Hq: int, Hkv: int, d: int) -> OperatorKey:
-    return OperatorKey("opattn_prefill", int(Hq), int(Hkv), int(d))
+    """The prefill-attention operator with Hq query heads, Hkv kv heads, head size d."""
+    return OperatorKey("opattn_prefill", (int(Hq), int(Hkv), int(d)))
+
+
+def gemm_key(k_in: int, n_out: int) -> OperatorKey:
+    """A token-wise projection: [tokens, k_in] x [k_in, n_out]."""
+    return OperatorKey("gemm", (int(k_in), int(n_out)))
 
 
 class ProfileStore:
@@ -158,6 +162,9 @@ class ProfileStore:
 
     def __len__(self) -> int:
         return len(self._profiles)
+
+    def __getitem__(self, key: OperatorKey) -> PiecewiseProfile:
+        return self._profiles[key]
 
     def get(self, key: OperatorKey, profile_fn) -> PiecewiseProfile:
         if key not in self._profiles:
@@ -179,7 +186,9 @@ class ProfileStore:
         s = cls()
         with open(path) as f:
             for e in json.load(f):
-                s._profiles[OperatorKey(**e["key"])] = PiecewiseProfile.from_dict(e["profile"])
+                k = e["key"]
+                key = OperatorKey(k["op"], tuple(k["shape"]), k["dtype"])
+                s._profiles[key] = PiecewiseProfile.from_dict(e["profile"])
         return s
 
 
@@ -201,14 +210,14 @@ class _Buffers:
         self.lse = torch.empty((n, Hq), dtype=torch.float32, device=device)
 
 
-def _time_plan_ms(plan, q, k, v, o, lse, scale, reps: int, warm_ms: float = 25.0, min_ms: float = 2.0) -> float:
-    """Median per-launch CUDA-event time (ms) of ``plan.run`` on the current stream.
+def time_callable_ms(fn, reps: int, warm_ms: float = 25.0, min_ms: float = 2.0) -> float:
+    """Median per-call CUDA-event time (ms) of ``fn`` launching work on the current stream.
 
-    The operator first runs back to back for ``warm_ms`` so the clocks leave
-    their idle state.  Each of the ``reps`` samples then times ``inner``
-    back-to-back launches between two events (``inner`` chosen so a sample
-    spans at least ``min_ms``), so the host's launch gap before a single short
-    launch is not counted.
+    ``fn`` first runs back to back for ``warm_ms`` so the clocks leave their
+    idle state.  Each of the ``reps`` samples then times ``inner`` back-to-back
+    calls between two events (``inner`` chosen so a sample spans at least
+    ``min_ms``), so the host's launch gap before a single short launch is not
+    counted.
     """
     import torch
     stream = torch.cuda.current_stream()
@@ -217,7 +226,7 @@ def _time_plan_ms(plan, q, k, v, o, lse, scale, reps: int, warm_ms: float = 25.0
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         for _ in range(inner):
-            plan.run(q, k, v, o, lse, scale, stream)
+            fn()
         b.record(stream)
         b.synchronize()
         return a.elapsed_time(b) / inner
@@ -228,6 +237,12 @@ def _time_plan_ms(plan, q, k, v, o, lse, scale, reps: int, warm_ms: float = 25.0
     while warm < warm_ms:
         warm += sample(inner) * inner
     return statistics.median(sample(inner) for _ in range(reps))
+
+
+def _time_plan_ms(plan, q, k, v, o, lse, scale, reps: int) -> float:
+    import torch
+    stream = torch.cuda.current_stream()
+    return time_callable_ms(lambda: plan.run(q, k, v, o, lse, scale, stream), reps)
 
 
 def n_sms() -> int:
@@ -263,6 +278,59 @@ def sm_budget_curve(w, ctas, reps: int = 5, device="cuda"):
         with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, max_ctas=n) as plan:
             out.append((plan.n_ctas, _time_plan_ms(plan, q, k, v, o, lse, w.scale, reps)))
     return out
+
+
+class GemmOperator:
+    """Times a bf16 token-wise projection (library matmul) for B prompts of L tokens."""
+
+    def __init__(self, k_in: int, n_out: int, max_tokens: int, device="cuda"):
+        import torch
+        g = torch.Generator(device=device)
+        g.manual_seed(0)
+        self.x = torch.randn((max_tokens, k_in), generator=g, device=device, dtype=torch.bfloat16)
+        self.w = torch.randn((k_in, n_out), generator=g, device=device, dtype=torch.bfloat16) * k_in ** -0.5
+        self.y = torch.empty((max_tokens, n_out), device=device, dtype=torch.bfloat16)
+
+    def measure(self, B: int, L: int, reps: int = 5) -> float:
+        import torch
+        m = B * L
+        return time_callable_ms(lambda: torch.matmul(self.x[:m], self.w, out=self.y[:m]), reps)
+
+
+def profile_operator(measure, n_train: int, rng, b_range=(1, 32), l_range=(128, 8192)) -> PiecewiseProfile:
+    """Sparse-sampling profile over (B, L) of any ``measure(B, L) -> ms``."""
+    pts = sample_points(n_train, rng, [b_range, l_range])
+    return PiecewiseProfile(pts, [measure(int(b), int(x)) for b, x in pts])
+
+
+def llama3_8b_layer_keys():
+    """The operators of one Llama-3-8B decoder layer that the provisioning study uses."""
+    return {"qkv_proj": gemm_key(4096, 6144), "attention": attention_key(32, 8, 128),
+            "o_proj": gemm_key(4096, 4096), "gate_up_proj": gemm_key(4096, 28672),
+            "down_proj": gemm_key(14336, 4096)}
+
+
+def build_store(n_train: int, seed: int = 0, b_range=(1, 32), l_range=(128, 8192), reps: int = 5) -> ProfileStore:
+    """Profiles of every distinct operator of Llama-3-8B's 32 layers (each measured once)."""
+    import torch
+    rng = np.random.default_rng(seed)
+    max_tokens = int(b_range[1] * l_range[1])
+    store = ProfileStore()
+
+    def profile(key):
+        if key.op == "opattn_prefill":
+            buf = _Buffers(max_tokens, *key.shape)
+            fn = lambda B, L: measure_ms(buf, B, L, reps=reps)
+        else:
+            g = GemmOperator(key.shape[0], key.shape[1], max_tokens)
+            fn = lambda B, L: g.measure(B, L, reps)
+        prof = profile_operator(fn, n_train, rng, b_range, l_range)
+        torch.cuda.empty_cache()
+        return prof
+
+    layers = [k for _ in range(32) for k in llama3_8b_layer_keys().values()]
+    store.profiles_for(layers, profile)
+    return store
 
 
 def profile_accuracy(n_train: int, n_test: int, seed: int = 0, key: OperatorKey = attention_key(32, 8, 128),
@@ -360,9 +428,16 @@ def main(argv=None):
     ap.add_argument("--reps", type=int, default=7)
     ap.add_argument("--out", default=None)
     ap.add_argument("--dump", default=None, help="write every measured point as JSON")
+    ap.add_argument("--store", default=None,
+                    help="only build the Llama-3-8B layer's operator profiles and save them here as JSON")
     args = ap.parse_args(argv)
     from . import build
     build.build()
+    if args.store:
+        store = build_store(args.train, args.seed, reps=args.reps)
+        store.save(args.store)
+        print(f"{len(store)} operator profiles ({len(store.measured)} measured) -> {args.store}")
+        return
     text = _report(args)
     if args.out:
         with open(args.out, "w") as f:

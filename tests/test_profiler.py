@@ -128,7 +128,7 @@ def test_structural_equivalence_profiles_each_shape_once(tmp_path):
     def fake_profile(key):
         calls.append(key)
         pts = np.array([[1, 128], [1, 8192], [32, 128], [32, 8192]], dtype=float)
-        return P.PiecewiseProfile(pts, key.Hq * attention_like(pts))
+        return P.PiecewiseProfile(pts, key.shape[0] * attention_like(pts))
 
     store = P.ProfileStore()
     llama3_70b = [P.attention_key(64, 8, 128)] * 80
@@ -140,12 +140,25 @@ def test_structural_equivalence_profiles_each_shape_once(tmp_path):
     store.profiles_for(llama31_8b, fake_profile)
     assert calls == [P.attention_key(64, 8, 128), P.attention_key(32, 8, 128)]
     assert len(store) == 2 and store.measured == calls
+    assert {k.name() for k in calls} == {"opattn_prefill[64, 8, 128]/bf16", "opattn_prefill[32, 8, 128]/bf16"}
     # a change of head grouping is a different operator
     assert P.attention_key(32, 32, 128) not in store
+    assert P.gemm_key(4096, 4096) not in store
+    store.get(P.gemm_key(4096, 4096), fake_profile)
     path = str(tmp_path / "profiles.json")
     store.save(path)
     back = P.ProfileStore.load(path)
-    assert len(back) == 2
+    assert len(back) == 3 and set(back._profiles) == set(store._profiles)
     q = [[7, 3000], [20, 500]]
     for key in calls:
         np.testing.assert_allclose(back.get(key, None).predict(q), store.get(key, None).predict(q), rtol=0)
+
+
+def test_llama3_8b_layer_has_five_distinct_operators():
+    keys = P.llama3_8b_layer_keys()
+    assert len(set(keys.values())) == 5
+    store = P.ProfileStore()
+    pts = np.array([[1, 128], [1, 8192], [32, 128], [32, 8192]], dtype=float)
+    store.profiles_for([k for _ in range(32) for k in keys.values()],
+                       lambda key: P.PiecewiseProfile(pts, attention_like(pts)))
+    assert len(store.measured) == 5          # 160 operator instances, 5 profiles
