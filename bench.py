@@ -3,6 +3,9 @@
 One step = one pass of the whole hot path (one persistent-kernel launch of
 opattn over the workload's ragged batch).  The headline workload is the
 Llama-3-70B-shaped layer (Hq 64, Hkv 8, d 128, 8 prompts x 4096 tokens).
+The decode workloads (--workload decode_*) time the decode kernel
+(opattn_decode) instead; it is bound by HBM, so its roofline is reported in
+GB/s of algorithmic traffic (q, k, v and o once, plus LSE).
 
 Metric: causal attention TFLOP/s, counting 4 * d * Hq FLOPs per visible
 (query, key) pair (2d for QK^T, 2d for PV; masked and skipped work, softmax
@@ -40,6 +43,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "prefill attention TFLOP/s (causal) and prompt tokens/s on 1 GB300; % BF16 peak"
+METRIC_DECODE = "decode attention TFLOP/s (causal) and HBM GB/s on 1 GB300; % measured HBM bandwidth"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -58,6 +62,11 @@ def visible_pairs(q_lens, k_lens) -> int:
 
 def causal_flops(w) -> int:
     return 4 * w.d * w.Hq * visible_pairs(w.q_lens, w.k_lens)
+
+
+def algorithmic_bytes(w) -> int:
+    """Bytes the operator must move at least: q, k, v read once, o and LSE written once."""
+    return 2 * w.d * (2 * w.total_q * w.Hq + 2 * w.total_k * w.Hkv) + 4 * w.total_q * w.Hq
 
 
 def row_flops(w, tokens, heads) -> int:
@@ -214,7 +223,7 @@ def run_reference(args, w):
     value = flops / secs / 1e12
     tokens_per_s = value * 1e12 / (causal_flops(w) / w.total_q)
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": args.gpus,
+        "impl": "reference", "metric": METRIC_DECODE if is_decode(w) else METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded N(0,1) bf16 inputs; counter-based generator)",
@@ -262,7 +271,9 @@ def run_ours(args, w):
     flops = causal_flops(w)
     stream = torch.cuda.current_stream(dev)
 
-    plan = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d)
+    decode = is_decode(w)
+    plan = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=decode)
+    one_shot = pkg.opattn_decode if decode else pkg.opattn_prefill
     for _ in range(max(args.warmup, 3)):
         plan.run(q, k, v, o, lse, w.scale, stream)
     torch.cuda.synchronize(dev)
@@ -305,7 +316,7 @@ def run_ours(args, w):
         dq.copy_(hq, non_blocking=True)
         dk.copy_(hk, non_blocking=True)
         dv.copy_(hv, non_blocking=True)
-        pkg.opattn_prefill(dq, dk, dv, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
+        one_shot(dq, dk, dv, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
         ho.copy_(o, non_blocking=True)
         hl.copy_(lse, non_blocking=True)
 
@@ -339,9 +350,20 @@ def run_ours(args, w):
     if rank == 0:
         peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
         peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-        traffic = recorded_traffic(w.name)
+        traffic = recorded_traffic(w.name, decode)
+        if decode:
+            hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+            gbs = algorithmic_bytes(w) / (kernel_ms / 1e3) / 1e9
+            roofline = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
+                        "traffic": traffic, "algorithmic_bytes": algorithmic_bytes(w),
+                        "peak_source": f"{peak_src} hbm_gbs"}
+        else:
+            roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                        "frac": achieved / peak, "traffic": traffic,
+                        "peak_source": f"{peak_src} bf16_tflops (burst)"}
         line = {
-            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "metric": METRIC_DECODE if decode else METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": elapsed_max / args.steps * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded N(0,1) bf16 q/k/v from a counter-based generator)",
@@ -352,9 +374,7 @@ def run_ours(args, w):
             "pct_bf16_peak_sustained": value / peak_sus,
             "kernel_ms": kernel_ms,
             "flops_per_step": flops,
-            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                         "frac": achieved / peak, "traffic": traffic,
-                         "peak_source": f"{peak_src} bf16_tflops (burst)"},
+            "roofline": roofline,
             "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "steps": e2e_steps},
             "cpu_baseline": cpu_base,
@@ -368,13 +388,18 @@ def run_ours(args, w):
     return 0
 
 
-def recorded_traffic(workload: str):
+def is_decode(w) -> bool:
+    from paper_2608_13499_gb300 import workloads as W
+    return any(f().name == w.name for f in W.DECODE.values())
+
+
+def recorded_traffic(workload: str, decode: bool = False):
     """DRAM bytes per launch from the committed ncu record, or None when the
     kernel sources changed since that capture (the counters no longer apply)."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
-    rev = kernel_revision()
+    rev = kernel_revision(decode)
     with open(path) as f:
         for line in f:
             parts = line.split()
@@ -383,11 +408,12 @@ def recorded_traffic(workload: str):
     return None
 
 
-def kernel_revision() -> str:
+def kernel_revision(decode: bool = False) -> str:
     """Hash of the kernel sources: traffic counters are only valid for the kernel they were taken on."""
     import hashlib
     h = hashlib.sha1()
-    for f in ("opattn_kernel.cu", "ptx.cuh", "opattn_internal.h"):
+    for f in ("opattn_decode.cu" if decode else "opattn_kernel.cu", "device_common.cuh", "ptx.cuh",
+              "opattn_internal.h"):
         with open(os.path.join(ROOT, "paper_2608_13499_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
@@ -400,14 +426,15 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama3_70b",
-                    help="tiny | llama3_8b | llama3_70b | bursty | chunked")
+                    help="tiny | llama3_8b | llama3_70b | bursty | chunked | decode_llama3_70b | "
+                         "decode_llama3_8b | decode_spec4_llama3_70b")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--reference-step-seconds", type=float, default=3.0)
     args = ap.parse_args(argv)
     from paper_2608_13499_gb300 import workloads as W
-    w = W.STANDARD[args.workload]()
+    w = {**W.STANDARD, **W.DECODE}[args.workload]()
     if args.impl == "reference":
         return run_reference(args, w)
     return run_ours(args, w)

@@ -173,6 +173,63 @@ OPATTN_API opattn_status opattn_schedule(const int32_t *cu_seqlens_q, const int3
                               int32_t *units, int64_t unit_capacity, int32_t *cta_offsets,
                               int64_t *n_units_out, int32_t *n_ctas_used);
 
+/*
+ * Decode-shaped batches.  A decode iteration (§3.1: each iteration after
+ * prefill produces one token per request, and its latency is held to the
+ * TBT objective) runs the same operator with one query token per sequence
+ * (a few with speculative tokens) over the sequence's whole cached key
+ * range.  opattn_decode computes exactly what opattn_prefill computes, with
+ * the same arguments, layouts, mask and outputs, with a kernel built for
+ * that shape: it is bound by reading K and V from HBM, cuts long key ranges
+ * into chunks processed in parallel (split-KV) and merges the chunks'
+ * partial results with their log-sum-exp weights inside the same launch.
+ *
+ * Supported shapes: d = 128, G = Hq / Hkv dividing 32 (1, 2, 4, 8, 16, 32),
+ * and Lq * G <= 32 for every sequence (e.g. G = 8: up to 4 query tokens per
+ * sequence); anything else returns OPATTN_ERR_UNSUPPORTED before any device
+ * work.  Lk may be anything, including 0 and Lk < Lq.
+ *
+ * Scratch: the one-shot call allocates its work list and the chunks'
+ * partial results (kDecCols x d fp32 per chunk, 16 KB) with cudaMallocAsync
+ * on `stream` and frees them there.  opattn_decode_checked additionally
+ * waits for the stream and reports a device timeout (flags as for
+ * opattn_prefill_checked).
+ */
+OPATTN_API opattn_status opattn_decode(const void *q, const void *k, const void *v, void *o, float *lse,
+                                       const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k, int32_t n_seq,
+                                       int32_t Hq, int32_t Hkv, int32_t d, float scale, void *stream);
+OPATTN_API opattn_status opattn_decode_checked(const void *q, const void *k, const void *v, void *o, float *lse,
+                                               const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                                               int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
+                                               void *stream, uint32_t flags);
+/*
+ * A plan for the decode kernel: same contract as opattn_plan_create, and the
+ * plan is run, queried and destroyed with opattn_plan_run / _info / _destroy.
+ * The plan owns the chunk partials, so two runs of one plan must not overlap
+ * (run them on one stream).  Each run zeroes the plan's merge counters with
+ * an asynchronous memset before the launch.
+ */
+OPATTN_API opattn_status opattn_decode_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
+                                                   const int32_t *cu_seqlens_k, int32_t n_seq, int32_t Hq,
+                                                   int32_t Hkv, int32_t d, int32_t max_ctas);
+/*
+ * Host-only decode scheduler (no GPU needed).  A unit is (sequence, kv head,
+ * chunk of 128-key tiles); a sequence's tiles are cut into equal chunks so
+ * that the CTAs get about six units each (at least 4 tiles per chunk), and
+ * units are packed onto CTAs longest first as in opattn_schedule.  Writes
+ * `units` as 12 int32 per unit:
+ *     {first packed query row, query tokens of the sequence, first packed key
+ *      row, Lk, kv head, first key tile of the chunk, tiles in the chunk,
+ *      partial slot (-1: the chunk is the whole sequence), merge group (-1),
+ *      chunk index, chunks of the (sequence, kv head), sequence index}
+ * and cta_offsets as opattn_schedule does.  Sequences with Lq = 0 get no unit.
+ */
+OPATTN_API opattn_status opattn_decode_schedule(const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                                                int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d,
+                                                int32_t n_ctas, int32_t *units, int64_t unit_capacity,
+                                                int32_t *cta_offsets, int64_t *n_units_out,
+                                                int32_t *n_ctas_used);
+
 #ifdef __cplusplus
 }
 #endif

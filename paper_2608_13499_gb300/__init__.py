@@ -1,4 +1,4 @@
-"""Python binding of libopattn (ragged causal GQA prefill attention on GB300).
+"""Python binding of libopattn (ragged causal GQA prefill and decode attention on GB300).
 
 Argument marshalling only: every step of the computation runs in the CUDA
 library behind the C ABI declared in ``include/opattn.h``.  PyTorch is used
@@ -27,6 +27,9 @@ OPATTN_FLAG_TEST_FORCE_TIMEOUT = 1
 OPATTN_NOALLOC_MAX_UNITS = 32768
 
 UNIT_FIELDS = ("q_tok0", "n_tok", "k_row0", "Lk", "qlim0", "kvh", "n_tiles", "seq")
+DEC_UNIT_FIELDS = ("q_tok0", "nq", "k_row0", "Lk", "kvh", "tile0", "n_tiles", "part", "group", "chunk", "n_chunks",
+                   "seq")
+DEC_COLS = 32
 
 _lock = threading.Lock()
 _lib = None
@@ -70,6 +73,15 @@ def load():
             lib.opattn_schedule.restype = ctypes.c_int
             lib.opattn_schedule.argtypes = [P, P, i32, i32, i32, i32, i32, P, i64, P,
                                             ctypes.POINTER(i64), ctypes.POINTER(i32)]
+            lib.opattn_decode.restype = ctypes.c_int
+            lib.opattn_decode.argtypes = [P, P, P, P, P, P, P, i32, i32, i32, i32, f32, P]
+            lib.opattn_decode_checked.restype = ctypes.c_int
+            lib.opattn_decode_checked.argtypes = [P, P, P, P, P, P, P, i32, i32, i32, i32, f32, P, u32]
+            lib.opattn_decode_plan_create.restype = ctypes.c_int
+            lib.opattn_decode_plan_create.argtypes = [ctypes.POINTER(P), P, P, i32, i32, i32, i32, i32]
+            lib.opattn_decode_schedule.restype = ctypes.c_int
+            lib.opattn_decode_schedule.argtypes = [P, P, i32, i32, i32, i32, i32, P, i64, P,
+                                                   ctypes.POINTER(i64), ctypes.POINTER(i32)]
             _lib = lib
     return _lib
 
@@ -146,36 +158,74 @@ def opattn_prefill_checked(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: i
                                              _stream_handle(stream), int(flags)))
 
 
-def opattn_schedule(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):
-    """C ``opattn_schedule`` (host only).  Returns (units [n, 8] int32, cta_offsets [n_ctas_used + 1])."""
+def _schedule(fn_name: str, width: int, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):
     lib = load()
+    fn = getattr(lib, fn_name)
     cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
     n_seq = len(cq) - 1
     n_units, n_used = ctypes.c_int64(0), ctypes.c_int32(0)
-    st = lib.opattn_schedule(_np_ptr(cq), _np_ptr(ck), n_seq, Hq, Hkv, d, n_ctas, None, 0, None,
-                             ctypes.byref(n_units), ctypes.byref(n_used))
+    st = fn(_np_ptr(cq), _np_ptr(ck), n_seq, Hq, Hkv, d, n_ctas, None, 0, None, ctypes.byref(n_units),
+            ctypes.byref(n_used))
     if st not in (OPATTN_OK, OPATTN_ERR_CAPACITY):
-        raise OpattnError(st, "opattn_schedule")
-    units = np.zeros((max(n_units.value, 1), 8), dtype=np.int32)
+        raise OpattnError(st, fn_name)
+    units = np.zeros((max(n_units.value, 1), width), dtype=np.int32)
     offs = np.zeros(max(n_used.value, 0) + 1, dtype=np.int32)
-    st = lib.opattn_schedule(_np_ptr(cq), _np_ptr(ck), n_seq, Hq, Hkv, d, n_ctas, _np_ptr(units),
-                             units.shape[0], _np_ptr(offs), ctypes.byref(n_units), ctypes.byref(n_used))
+    st = fn(_np_ptr(cq), _np_ptr(ck), n_seq, Hq, Hkv, d, n_ctas, _np_ptr(units), units.shape[0], _np_ptr(offs),
+            ctypes.byref(n_units), ctypes.byref(n_used))
     if st != OPATTN_OK:
-        raise OpattnError(st, "opattn_schedule")
+        raise OpattnError(st, fn_name)
     return units[:n_units.value], offs
 
 
-class Plan:
-    """C ``opattn_plan_*``: a work list built and uploaded once, run many times."""
+def opattn_schedule(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):
+    """C ``opattn_schedule`` (host only).  Returns (units [n, 8] int32, cta_offsets [n_ctas_used + 1])."""
+    return _schedule("opattn_schedule", len(UNIT_FIELDS), cu_seqlens_q, cu_seqlens_k, Hq, Hkv, d, n_ctas)
 
-    def __init__(self, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, max_ctas: int = 0):
+
+def opattn_decode_schedule(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):
+    """C ``opattn_decode_schedule`` (host only).  Returns (units [n, 12] int32, cta_offsets)."""
+    return _schedule("opattn_decode_schedule", len(DEC_UNIT_FIELDS), cu_seqlens_q, cu_seqlens_k, Hq, Hkv, d,
+                     n_ctas)
+
+
+def opattn_decode(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int,
+                  scale: float, stream=None, *, check: bool = True) -> int:
+    """C ``opattn_decode``: the arguments and results of opattn_prefill, for batches
+    with few query tokens per sequence (Lq * Hq / Hkv <= 32, d = 128)."""
+    cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
+    st = load().opattn_decode(_dptr(q), _dptr(k), _dptr(v), _dptr(o), _dptr(lse), _np_ptr(cq), _np_ptr(ck),
+                              int(n_seq), int(Hq), int(Hkv), int(d), float(scale), _stream_handle(stream))
+    if check and st != OPATTN_OK:
+        raise OpattnError(st, "opattn_decode")
+    return st
+
+
+def opattn_decode_checked(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int,
+                          scale: float, stream=None, flags: int = 0) -> int:
+    """C ``opattn_decode_checked`` (synchronous; returns the status code)."""
+    cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
+    return int(load().opattn_decode_checked(_dptr(q), _dptr(k), _dptr(v), _dptr(o), _dptr(lse), _np_ptr(cq),
+                                            _np_ptr(ck), int(n_seq), int(Hq), int(Hkv), int(d), float(scale),
+                                            _stream_handle(stream), int(flags)))
+
+
+class Plan:
+    """C ``opattn_plan_*``: a work list built and uploaded once, run many times.
+
+    ``decode=True`` builds the plan with ``opattn_decode_plan_create`` (the
+    decode kernel); run, info and destroy are shared.
+    """
+
+    def __init__(self, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, max_ctas: int = 0,
+                 decode: bool = False):
         lib = load()
         cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
         self._h = ctypes.c_void_p()
-        st = lib.opattn_plan_create(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1, Hq, Hkv, d,
-                                    max_ctas)
+        self.decode = decode
+        create = lib.opattn_decode_plan_create if decode else lib.opattn_plan_create
+        st = create(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1, Hq, Hkv, d, max_ctas)
         if st != OPATTN_OK:
-            raise OpattnError(st, "opattn_plan_create")
+            raise OpattnError(st, "opattn_decode_plan_create" if decode else "opattn_plan_create")
         n_units, n_ctas = ctypes.c_int64(0), ctypes.c_int32(0)
         lib.opattn_plan_info(self._h, ctypes.byref(n_units), ctypes.byref(n_ctas))
         self.n_units, self.n_ctas = n_units.value, n_ctas.value
@@ -217,4 +267,17 @@ def prefill(q, k, v, cu_seqlens_q, cu_seqlens_k, scale: float | None = None, str
     n_seq = len(cu_seqlens_q) - 1
     opattn_prefill(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d,
                    scale if scale is not None else d ** -0.5, stream)
+    return o, lse
+
+
+def decode(q, k, v, cu_seqlens_q, cu_seqlens_k, scale: float | None = None, stream=None):
+    """Allocate O and LSE with torch and run opattn_decode on CUDA tensors q [Tq,Hq,d], k/v [Tk,Hkv,d]."""
+    import torch
+    Tq, Hq, d = q.shape
+    Hkv = k.shape[1]
+    o = torch.empty((Tq, Hq, d), dtype=torch.bfloat16, device=q.device)
+    lse = torch.empty((Tq, Hq), dtype=torch.float32, device=q.device)
+    n_seq = len(cu_seqlens_q) - 1
+    opattn_decode(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d,
+                  scale if scale is not None else d ** -0.5, stream)
     return o, lse

@@ -1,4 +1,4 @@
-"""Builds libopattn.so in-tree with nvcc for sm_103a (no cmake, two translation units)."""
+"""Builds libopattn.so in-tree with nvcc for sm_103a (no cmake; the translation units compile in parallel)."""
 from __future__ import annotations
 
 import os
@@ -15,8 +15,8 @@ LIB = os.path.join(PKG, "libopattn.so")
 BUILD_DIR = os.path.join(PKG, "_build")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["opattn_kernel.cu", "opattn_api.cpp", "opattn_noalloc.cu"]
-DEPS = ["ptx.cuh", "opattn_internal.h"]
+SOURCES = ["opattn_kernel.cu", "opattn_decode.cu", "opattn_api.cpp", "opattn_noalloc.cu"]
+DEPS = ["ptx.cuh", "opattn_internal.h", "device_common.cuh"]
 
 
 def nvcc() -> str:
@@ -35,7 +35,7 @@ def _stale() -> bool:
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile both translation units in parallel and link libopattn.so; returns its path."""
+    """Compile the translation units in parallel and link libopattn.so; returns its path."""
     if not force and not _stale():
         return LIB
     os.makedirs(BUILD_DIR, exist_ok=True)

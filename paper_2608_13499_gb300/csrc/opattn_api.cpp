@@ -76,12 +76,60 @@ struct Schedule {
     int32_t n_cta = 0;
 };
 
+// Longest-processing-time packing: units are bucket-sorted by cost, longest
+// first (stable: enumeration order within a cost), and each goes to the CTA
+// with the least cost so far (ties: lower CTA index); makespan within 4/3 of
+// optimal.  Writes the units grouped by CTA and the CSR offsets.
+template <class U, class CostFn>
+void lpt_pack(const std::vector<U>& all, int32_t max_cost, int32_t max_ctas, CostFn cost, std::vector<U>* units,
+              std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
+    const int64_t n = static_cast<int64_t>(all.size());
+    units->clear();
+    cta_off->clear();
+    *n_cta_out = 0;
+    if (n == 0) return;
+    const int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(std::max<int32_t>(max_ctas, 1), n));
+
+    std::vector<int64_t> count(static_cast<size_t>(max_cost) + 2, 0);
+    for (const U& u : all) ++count[static_cast<size_t>(max_cost - cost(u))];
+    int64_t acc = 0;
+    for (auto& c : count) {
+        const int64_t t = c;
+        c = acc;
+        acc += t;
+    }
+    std::vector<int64_t> order(static_cast<size_t>(n));
+    for (int64_t i = 0; i < n; ++i) order[static_cast<size_t>(count[static_cast<size_t>(max_cost - cost(all[static_cast<size_t>(i)]))]++)] = i;
+
+    using Slot = std::pair<int64_t, int32_t>;
+    std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> heap;
+    for (int32_t c = 0; c < n_cta; ++c) heap.push({0, c});
+    std::vector<int32_t> owner(static_cast<size_t>(n));
+    std::vector<int32_t> per_cta(static_cast<size_t>(n_cta), 0);
+    for (int64_t i = 0; i < n; ++i) {
+        Slot sl = heap.top();
+        heap.pop();
+        owner[static_cast<size_t>(i)] = sl.second;
+        ++per_cta[static_cast<size_t>(sl.second)];
+        sl.first += cost(all[static_cast<size_t>(order[static_cast<size_t>(i)])]);
+        heap.push(sl);
+    }
+    cta_off->assign(static_cast<size_t>(n_cta) + 1, 0);
+    for (int32_t c = 0; c < n_cta; ++c)
+        (*cta_off)[static_cast<size_t>(c) + 1] = (*cta_off)[static_cast<size_t>(c)] + per_cta[static_cast<size_t>(c)];
+    std::vector<int32_t> fill(cta_off->begin(), cta_off->end() - 1);
+    units->resize(static_cast<size_t>(n));
+    for (int64_t i = 0; i < n; ++i) {
+        const int32_t c = owner[static_cast<size_t>(i)];
+        (*units)[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = all[static_cast<size_t>(order[static_cast<size_t>(i)])];
+    }
+    *n_cta_out = n_cta;
+}
+
 // Units are (sequence, kv head, block of 2 * TPB query tokens).  Cost is the
 // number of key tiles the block visits after whole tiles above the causal
-// diagonal are skipped, plus one for the Q load and the epilogue.  Units are
-// bucket-sorted by cost, longest first, and each goes to the CTA with the
-// least cost so far (longest-processing-time greedy; makespan within 4/3 of
-// optimal).
+// diagonal are skipped, plus one for the Q load and the epilogue; units are
+// packed onto CTAs longest first.
 void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out) {
     const int32_t tpu = 2 * g.TPB;
     std::vector<UnitRec> all;
@@ -110,49 +158,8 @@ void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g,
             }
         }
     }
-    const int64_t n = static_cast<int64_t>(all.size());
-    out->units.clear();
-    out->cta_off.clear();
-    out->n_cta = 0;
-    if (n == 0) return;
-    const int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(std::max<int32_t>(max_ctas, 1), n));
-
-    // counting sort by cost, descending (stable: sequence order within a cost)
-    std::vector<int64_t> count(static_cast<size_t>(max_cost) + 2, 0);
-    for (const UnitRec& u : all) ++count[static_cast<size_t>(max_cost - (u.n_tiles + 1))];
-    int64_t acc = 0;
-    for (auto& c : count) {
-        const int64_t t = c;
-        c = acc;
-        acc += t;
-    }
-    std::vector<int64_t> order(static_cast<size_t>(n));
-    for (int64_t i = 0; i < n; ++i) order[static_cast<size_t>(count[static_cast<size_t>(max_cost - (all[i].n_tiles + 1))]++)] = i;
-
-    // greedy: next unit to the least-loaded CTA (ties: lower CTA index)
-    using Slot = std::pair<int64_t, int32_t>;
-    std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> heap;
-    for (int32_t c = 0; c < n_cta; ++c) heap.push({0, c});
-    std::vector<int32_t> owner(static_cast<size_t>(n));
-    std::vector<int32_t> per_cta(static_cast<size_t>(n_cta), 0);
-    for (int64_t i = 0; i < n; ++i) {
-        Slot sl = heap.top();
-        heap.pop();
-        const UnitRec& u = all[static_cast<size_t>(order[static_cast<size_t>(i)])];
-        owner[static_cast<size_t>(i)] = sl.second;
-        ++per_cta[static_cast<size_t>(sl.second)];
-        sl.first += u.n_tiles + 1;
-        heap.push(sl);
-    }
-    out->cta_off.assign(static_cast<size_t>(n_cta) + 1, 0);
-    for (int32_t c = 0; c < n_cta; ++c) out->cta_off[static_cast<size_t>(c) + 1] = out->cta_off[static_cast<size_t>(c)] + per_cta[static_cast<size_t>(c)];
-    std::vector<int32_t> fill(out->cta_off.begin(), out->cta_off.end() - 1);
-    out->units.resize(static_cast<size_t>(n));
-    for (int64_t i = 0; i < n; ++i) {
-        const int32_t c = owner[static_cast<size_t>(i)];
-        out->units[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = all[static_cast<size_t>(order[static_cast<size_t>(i)])];
-    }
-    out->n_cta = n_cta;
+    lpt_pack(all, max_cost, max_ctas, [](const UnitRec& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
+             &out->n_cta);
 }
 
 // Device work area: [cta_off (n_cta + 1) | pad to 32 B | units | status].
@@ -341,6 +348,179 @@ opattn_status prefill_noalloc_impl(const void* q, const void* k, const void* v, 
     return launch_prefill(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
 }
 
+// ------------------------------------------------------------------ decode
+
+// Additional checks of the decode kernel: d = 128, G divides kDecCols, and
+// every sequence's G * Lq query (token, head) pairs fit the kDecCols columns.
+opattn_status check_decode_geometry(const int32_t* cu_q, const Geometry& g) {
+    if (g.d != kDecHeadDim) return OPATTN_ERR_UNSUPPORTED;
+    if (kDecCols % g.G != 0) return OPATTN_ERR_UNSUPPORTED;
+    for (int32_t s = 0; s < g.n_seq; ++s)
+        if (static_cast<int64_t>(cu_q[s + 1] - cu_q[s]) * g.G > kDecCols) return OPATTN_ERR_UNSUPPORTED;
+    return OPATTN_OK;
+}
+
+struct DecodeSchedule {
+    std::vector<DecUnit> units;    // grouped by CTA, longest first within a CTA
+    std::vector<int32_t> cta_off;  // n_cta + 1
+    int32_t n_cta = 0;
+    int32_t n_groups = 0;          // split (sequence, kv head) pairs: one merge counter each
+    int32_t n_parts = 0;           // partial (O, LSE) slots
+    int32_t chunk_tiles = 0;       // target key tiles per chunk
+    int32_t max_cols = 0;          // largest G * Lq over the batch
+};
+
+constexpr int32_t kDecMinChunkTiles = 4;  // 512 keys: below this a chunk's fixed costs dominate
+constexpr int32_t kDecChunksPerCta = 6;   // aim for about this many units per CTA
+
+// Units are (sequence, kv head, chunk of key tiles).  A sequence's key tiles
+// are cut into equal chunks of about chunk_tiles tiles, with chunk_tiles
+// sized so that the CTAs get about kDecChunksPerCta units each; the units
+// are packed onto CTAs longest first (cost = tiles + 1).
+void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas,
+                           DecodeSchedule* out) {
+    int64_t total_tiles = 0;
+    for (int32_t s = 0; s < g.n_seq; ++s)
+        if (cu_q[s + 1] > cu_q[s]) total_tiles += static_cast<int64_t>((cu_k[s + 1] - cu_k[s] + kBlockN - 1) / kBlockN) * g.Hkv;
+    const int64_t ctas = std::max<int32_t>(max_ctas, 1);
+    const int64_t per_cta = (total_tiles + ctas - 1) / ctas;
+    const int32_t chunk = static_cast<int32_t>(
+        std::max<int64_t>(kDecMinChunkTiles, (per_cta + kDecChunksPerCta - 1) / kDecChunksPerCta));
+    std::vector<DecUnit> all;
+    int32_t max_cost = 0, n_groups = 0, n_parts = 0;
+    for (int32_t s = 0; s < g.n_seq; ++s) {
+        const int32_t Lq = cu_q[s + 1] - cu_q[s];
+        if (Lq == 0) continue;
+        const int32_t Lk = cu_k[s + 1] - cu_k[s];
+        const int32_t n_t = (Lk + kBlockN - 1) / kBlockN;
+        const int32_t n_chunks = n_t == 0 ? 1 : (n_t + chunk - 1) / chunk;
+        for (int32_t h = 0; h < g.Hkv; ++h) {
+            const int32_t group = n_chunks > 1 ? n_groups++ : -1;
+            const int32_t part0 = n_chunks > 1 ? n_parts : -1;
+            if (n_chunks > 1) n_parts += n_chunks;
+            for (int32_t c = 0; c < n_chunks; ++c) {
+                const int32_t t0 = static_cast<int32_t>(static_cast<int64_t>(c) * n_t / n_chunks);
+                const int32_t t1 = static_cast<int32_t>(static_cast<int64_t>(c + 1) * n_t / n_chunks);
+                DecUnit u;
+                u.q_tok0 = cu_q[s];
+                u.nq = Lq;
+                u.k_row0 = cu_k[s];
+                u.Lk = Lk;
+                u.kvh = h;
+                u.tile0 = t0;
+                u.n_tiles = t1 - t0;
+                u.part = n_chunks > 1 ? part0 + c : -1;
+                u.group = group;
+                u.chunk = c;
+                u.n_chunks = n_chunks;
+                u.seq = s;
+                max_cost = std::max(max_cost, u.n_tiles + 1);
+                all.push_back(u);
+            }
+        }
+    }
+    lpt_pack(all, max_cost, max_ctas, [](const DecUnit& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
+             &out->n_cta);
+    out->n_groups = n_groups;
+    out->n_parts = n_parts;
+    out->chunk_tiles = chunk;
+    int32_t max_cols = 1;
+    for (int32_t s = 0; s < g.n_seq; ++s) max_cols = std::max(max_cols, (cu_q[s + 1] - cu_q[s]) * g.G);
+    out->max_cols = max_cols;
+}
+
+// Device work area: [cta_off | pad 32 | units | counters (n_groups) | status |
+// pad 256 | part_lse (n_parts x kDecCols) | part_o (n_parts x kDecCols x d)].
+// The counters and the status word are contiguous and zeroed before every
+// launch.
+struct DecodeLayout {
+    size_t off_units, off_counters, off_status, off_part_lse, off_part_o, bytes, upload_bytes, zero_bytes;
+};
+DecodeLayout decode_layout(const DecodeSchedule& s) {
+    DecodeLayout w;
+    w.off_units = (s.cta_off.size() * sizeof(int32_t) + 31) / 32 * 32;
+    w.off_counters = w.off_units + s.units.size() * sizeof(DecUnit);
+    w.off_status = w.off_counters + static_cast<size_t>(s.n_groups) * sizeof(int32_t);
+    w.upload_bytes = w.off_counters;
+    w.zero_bytes = w.off_status + sizeof(int32_t) - w.off_counters;
+    w.off_part_lse = (w.off_status + sizeof(int32_t) + 255) / 256 * 256;
+    w.off_part_o = w.off_part_lse + (static_cast<size_t>(s.n_parts) * kDecCols * sizeof(float) + 255) / 256 * 256;
+    w.bytes = w.off_part_o + static_cast<size_t>(s.n_parts) * kDecCols * kDecHeadDim * sizeof(float);
+    return w;
+}
+void pack_decode_upload(const DecodeSchedule& s, const DecodeLayout& w, uint8_t* dst) {
+    std::memset(dst, 0, w.upload_bytes);
+    std::memcpy(dst, s.cta_off.data(), s.cta_off.size() * sizeof(int32_t));
+    std::memcpy(dst + w.off_units, s.units.data(), s.units.size() * sizeof(DecUnit));
+}
+DecodeLaunchArgs make_decode_args(const void* q, const void* k, const void* v, void* o, float* lse,
+                                  const Geometry& g, float scale, uint8_t* work, const DecodeLayout& w,
+                                  int32_t n_cta, int32_t max_cols, uint32_t flags) {
+    DecodeLaunchArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.o = o;
+    a.lse = lse;
+    a.total_q = g.total_q;
+    a.total_k = g.total_k;
+    a.Hq = g.Hq;
+    a.Hkv = g.Hkv;
+    a.scale = scale;
+    a.units = reinterpret_cast<const DecUnit*>(work + w.off_units);
+    a.cta_off = reinterpret_cast<const int32_t*>(work);
+    a.n_cta = n_cta;
+    a.max_cols = max_cols;
+    a.counters = reinterpret_cast<int32_t*>(work + w.off_counters);
+    a.part_lse = reinterpret_cast<float*>(work + w.off_part_lse);
+    a.part_o = reinterpret_cast<float*>(work + w.off_part_o);
+    a.status = reinterpret_cast<int32_t*>(work + w.off_status);
+    a.flags = flags;
+    return a;
+}
+
+opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
+                          const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
+                          cudaStream_t stream, uint32_t flags, bool checked) {
+    Geometry g;
+    opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    st = check_decode_geometry(cu_q, g);
+    if (st != OPATTN_OK) return st;
+    if (g.total_q == 0) return OPATTN_OK;
+    st = check_tensors(q, k, v, o, lse, scale, g);
+    if (st != OPATTN_OK) return st;
+    const int sms = device_sm_count();
+    if (sms <= 0) return OPATTN_ERR_CUDA;
+
+    DecodeSchedule sch;
+    build_decode_schedule(cu_q, cu_k, g, sms, &sch);
+    const DecodeLayout w = decode_layout(sch);
+    Staging* stg = staging_acquire(w.upload_bytes);
+    if (!stg) return OPATTN_ERR_CUDA;
+    pack_decode_upload(sch, w, static_cast<uint8_t*>(stg->host));
+    void* work = nullptr;
+    if (cudaMallocAsync(&work, w.bytes, stream) != cudaSuccess) {
+        staging_release(stg, stream);
+        return OPATTN_ERR_CUDA;
+    }
+    uint8_t* wb = static_cast<uint8_t*>(work);
+    bool ok = cudaMemcpyAsync(wb, stg->host, w.upload_bytes, cudaMemcpyHostToDevice, stream) == cudaSuccess;
+    ok = ok && cudaMemsetAsync(wb + w.off_counters, 0, w.zero_bytes, stream) == cudaSuccess;
+    staging_release(stg, stream);
+    int32_t dev_status = 0;
+    if (ok) ok = launch_decode(make_decode_args(q, k, v, o, lse, g, scale, wb, w, sch.n_cta, sch.max_cols, flags), stream) == 0;
+    if (ok && checked) {
+        ok = cudaMemcpyAsync(&dev_status, wb + w.off_status, sizeof(int32_t), cudaMemcpyDeviceToHost, stream) ==
+             cudaSuccess;
+        ok = ok && cudaStreamSynchronize(stream) == cudaSuccess;
+    }
+    cudaFreeAsync(work, stream);
+    if (!ok) return OPATTN_ERR_CUDA;
+    if (checked && dev_status != kDevOk) return OPATTN_ERR_TIMEOUT;
+    return OPATTN_OK;
+}
+
 }  // namespace
 }  // namespace opattn
 
@@ -348,8 +528,11 @@ using namespace opattn;
 
 struct opattn_plan {
     Geometry g;
-    Schedule sch;
+    bool decode = false;
+    Schedule sch;          // prefill plans
     WorkLayout w;
+    DecodeSchedule dsch;   // decode plans
+    DecodeLayout dw;
     int device = 0;
     void* work = nullptr;
 };
@@ -362,7 +545,9 @@ const char* opattn_status_string(int32_t status) {
     switch (status) {
         case OPATTN_OK: return "ok";
         case OPATTN_ERR_INVALID_ARG: return "invalid argument";
-        case OPATTN_ERR_UNSUPPORTED: return "unsupported configuration (head dim must be 64 or 128, Hq/Hkv <= 128)";
+        case OPATTN_ERR_UNSUPPORTED:
+            return "unsupported configuration (prefill: head dim 64 or 128, Hq/Hkv <= 128; decode: head dim 128, "
+                   "Hq/Hkv divides 32, Lq * Hq/Hkv <= 32 per sequence)";
         case OPATTN_ERR_MISALIGNED: return "misaligned pointer (q/k/v/o need 16 bytes, lse 4 bytes)";
         case OPATTN_ERR_CUDA: return "CUDA runtime error";
         case OPATTN_ERR_TIMEOUT: return "device wait timed out";
@@ -440,9 +625,17 @@ opattn_status opattn_plan_run(const opattn_plan* plan, const void* q, const void
     if (plan->g.total_q == 0) return OPATTN_OK;
     opattn_status st = check_tensors(q, k, v, o, lse, scale, plan->g);
     if (st != OPATTN_OK) return st;
-    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, static_cast<uint8_t*>(plan->work), plan->w,
-                                   plan->sch.n_cta, 0u);
-    return launch_prefill(a, static_cast<cudaStream_t>(stream)) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+    uint8_t* work = static_cast<uint8_t*>(plan->work);
+    const cudaStream_t st_ = static_cast<cudaStream_t>(stream);
+    if (plan->decode) {
+        if (cudaMemsetAsync(work + plan->dw.off_counters, 0, plan->dw.zero_bytes, st_) != cudaSuccess)
+            return OPATTN_ERR_CUDA;
+        const DecodeLaunchArgs a =
+            make_decode_args(q, k, v, o, lse, plan->g, scale, work, plan->dw, plan->dsch.n_cta, plan->dsch.max_cols, 0u);
+        return launch_decode(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+    }
+    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, work, plan->w, plan->sch.n_cta, 0u);
+    return launch_prefill(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
 }
 
 opattn_status opattn_plan_destroy(opattn_plan* plan) {
@@ -462,8 +655,8 @@ opattn_status opattn_plan_destroy(opattn_plan* plan) {
 
 opattn_status opattn_plan_info(const opattn_plan* plan, int64_t* n_units, int32_t* n_ctas) {
     if (!plan) return OPATTN_ERR_INVALID_ARG;
-    if (n_units) *n_units = static_cast<int64_t>(plan->sch.units.size());
-    if (n_ctas) *n_ctas = plan->sch.n_cta;
+    if (n_units) *n_units = static_cast<int64_t>(plan->decode ? plan->dsch.units.size() : plan->sch.units.size());
+    if (n_ctas) *n_ctas = plan->decode ? plan->dsch.n_cta : plan->sch.n_cta;
     return OPATTN_OK;
 }
 
@@ -482,6 +675,88 @@ opattn_status opattn_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seq
     if (!sch.units.empty() && (!units || !cta_offsets)) return OPATTN_ERR_INVALID_ARG;
     if (!sch.units.empty()) {
         std::memcpy(units, sch.units.data(), sch.units.size() * sizeof(UnitRec));
+        std::memcpy(cta_offsets, sch.cta_off.data(), sch.cta_off.size() * sizeof(int32_t));
+    }
+    return OPATTN_OK;
+}
+
+opattn_status opattn_decode(const void* q, const void* k, const void* v, void* o, float* lse,
+                            const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq, int32_t Hq,
+                            int32_t Hkv, int32_t d, float scale, void* stream) {
+    return decode_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
+                       static_cast<cudaStream_t>(stream), 0u, false);
+}
+
+opattn_status opattn_decode_checked(const void* q, const void* k, const void* v, void* o, float* lse,
+                                    const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
+                                    int32_t Hq, int32_t Hkv, int32_t d, float scale, void* stream, uint32_t flags) {
+    if (flags & ~OPATTN_FLAG_TEST_FORCE_TIMEOUT) return OPATTN_ERR_INVALID_ARG;
+    const uint32_t kflags = (flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u;
+    return decode_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
+                       static_cast<cudaStream_t>(stream), kflags, true);
+}
+
+opattn_status opattn_decode_plan_create(opattn_plan** plan, const int32_t* cu_seqlens_q,
+                                        const int32_t* cu_seqlens_k, int32_t n_seq, int32_t Hq, int32_t Hkv,
+                                        int32_t d, int32_t max_ctas) {
+    if (!plan) return OPATTN_ERR_INVALID_ARG;
+    *plan = nullptr;
+    if (max_ctas < 0) return OPATTN_ERR_INVALID_ARG;
+    Geometry g;
+    opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    st = check_decode_geometry(cu_seqlens_q, g);
+    if (st != OPATTN_OK) return st;
+    opattn_plan* p = new opattn_plan;
+    p->g = g;
+    p->decode = true;
+    if (cudaGetDevice(&p->device) != cudaSuccess) {
+        delete p;
+        return OPATTN_ERR_CUDA;
+    }
+    if (g.total_q > 0) {
+        const int sms = device_sm_count();
+        if (sms <= 0) {
+            delete p;
+            return OPATTN_ERR_CUDA;
+        }
+        const int32_t cap = max_ctas > 0 ? std::min(max_ctas, sms) : sms;
+        build_decode_schedule(cu_seqlens_q, cu_seqlens_k, g, cap, &p->dsch);
+        p->dw = decode_layout(p->dsch);
+        std::vector<uint8_t> host(p->dw.upload_bytes, 0);
+        pack_decode_upload(p->dsch, p->dw, host.data());
+        if (cudaMalloc(&p->work, p->dw.bytes) != cudaSuccess) {
+            delete p;
+            return OPATTN_ERR_CUDA;
+        }
+        if (cudaMemcpy(p->work, host.data(), p->dw.upload_bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+            cudaFree(p->work);
+            delete p;
+            return OPATTN_ERR_CUDA;
+        }
+    }
+    *plan = p;
+    return OPATTN_OK;
+}
+
+opattn_status opattn_decode_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
+                                     int32_t Hq, int32_t Hkv, int32_t d, int32_t n_ctas, int32_t* units,
+                                     int64_t unit_capacity, int32_t* cta_offsets, int64_t* n_units_out,
+                                     int32_t* n_ctas_used) {
+    if (n_ctas <= 0 || !n_units_out || !n_ctas_used) return OPATTN_ERR_INVALID_ARG;
+    Geometry g;
+    opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
+    if (st != OPATTN_OK) return st;
+    st = check_decode_geometry(cu_seqlens_q, g);
+    if (st != OPATTN_OK) return st;
+    DecodeSchedule sch;
+    build_decode_schedule(cu_seqlens_q, cu_seqlens_k, g, n_ctas, &sch);
+    *n_units_out = static_cast<int64_t>(sch.units.size());
+    *n_ctas_used = sch.n_cta;
+    if (static_cast<int64_t>(sch.units.size()) > unit_capacity) return OPATTN_ERR_CAPACITY;
+    if (!sch.units.empty() && (!units || !cta_offsets)) return OPATTN_ERR_INVALID_ARG;
+    if (!sch.units.empty()) {
+        std::memcpy(units, sch.units.data(), sch.units.size() * sizeof(DecUnit));
         std::memcpy(cta_offsets, sch.cta_off.data(), sch.cta_off.size() * sizeof(int32_t));
     }
     return OPATTN_OK;

@@ -1,0 +1,630 @@
+// opattn_decode.cu -- persistent sm_103a kernel for decode-shaped causal GQA
+// attention: few query tokens per sequence over a long key range (the decode
+// iterations of §3.1, whose per-token latency is the TBT objective).
+//
+// It computes the same bottom-right-aligned causal softmax attention as the
+// prefill kernel.  With G query heads per kv head and Lq <= 32 / G query
+// tokens, the (token, head) pairs of one kv head are too few to fill an
+// M = 128 tile, so the products are transposed:
+//   S^T (128 keys x 32 columns)  = K_tile (128 x d)      . Q^T (d x 32)
+//   O^T (d x 32 columns)        += V_tile^T (d x 128 keys) . P^T (128 x 32)
+// Both are tcgen05 MMAs with M = 128 (keys, then channels of d) and N = 32,
+// so every TMEM lane carries work even at G = 8, Lq = 1.  Column c is query
+// token c / G, head c % G of the kv head.  The kernel is bound by HBM: each
+// K/V byte is read once and feeds 2 * G * Lq flops.
+//
+// Softmax runs per column over the keys of a tile, one key per thread of the
+// softmax warpgroup (one TMEM lane each).  The subtraction base of a column
+// is the exact maximum of the chunk's first tile and is reused while no
+// score exceeds it by more than 2^kRebaseSlack; a larger score makes the
+// warpgroup take the tile's exact maximum and rescale the running sums and
+// the O accumulator.  Long key ranges are split into chunks (split-KV); a
+// chunk writes its normalised partial O and its log2-domain LSE, and the
+// last chunk of a (sequence, kv head) to finish merges the partials with
+// LSE weights.
+//
+// CTA layout (192 threads, one CTA per SM, persistent over its unit list):
+//   warps 0-3  softmax / epilogue / merge (thread t = TMEM lane t)
+//   warp 4     TMA producer: Q^T of the unit, then K_j and V_j
+//   warp 5     TMEM owner + MMA issuer (whole warp, one elected lane issues)
+// TMEM (128 columns): S0 | S1 (32 fp32 columns each) | O (32 columns).
+//
+// MMA order (tiles counted across the CTA's units as g):
+//   S(0), S(1), then per tile: wait P(g), PV(g), S(g + 2)
+// S(g + 2) reuses the S buffer of tile g only after PV(g), i.e. after the
+// softmax warps have read S(g) and written P(g).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "device_common.cuh"
+#include "opattn_internal.h"
+#include "ptx.cuh"
+
+namespace opattn {
+namespace {
+
+constexpr int D = kDecHeadDim;
+constexpr int NC = kDecCols;
+constexpr int kTile = 128;  // keys per K/V tile
+constexpr int kThreadsDec = 192;
+constexpr int kWarpProducerDec = 4;
+constexpr int kWarpMmaDec = 5;
+constexpr uint32_t kBarWG = 1;        // named barrier of the softmax warpgroup
+constexpr uint32_t kWGThreads = 128;
+// A score may exceed its column's subtraction base by up to 2^24 in the
+// exponential before the base is moved: fp32 sums of up to 2^31 keys and the
+// fp32 O accumulator stay far from overflow.
+constexpr float kRebaseSlack = 24.f;
+constexpr float kLn2Dec = 0.693147180559945309f;
+constexpr float kLog2eDec = 1.442695040888963407f;
+
+struct DCfg {
+    static constexpr int kQBytes = NC * D * 2;       // Q^T operand: NC rows x d, two 64-channel blocks
+    static constexpr int kSlotBytes = kTile * D * 2;  // one K or V tile
+    static constexpr int kKSlots = 3;
+    static constexpr int kVSlots = 3;
+    static constexpr int kPBytes = NC * kTile * 2;    // P^T operand: NC rows x 128 keys
+    static constexpr int kQOff = 0;                   // two Q buffers (unit parity)
+    static constexpr int kKOff = 2 * kQBytes;
+    static constexpr int kVOff = kKOff + kKSlots * kSlotBytes;
+    static constexpr int kPOff = kVOff + kVSlots * kSlotBytes;  // two P buffers (tile parity)
+    static constexpr int kRedOff = kPOff + 2 * kPBytes;         // two [4 warps][32] float buffers
+    static constexpr int kRedBytes = 2 * 4 * 32 * 4;
+    static constexpr int kBarOff = kRedOff + kRedBytes;
+    static constexpr int kBarKFull = 0;
+    static constexpr int kBarKEmpty = kKSlots;
+    static constexpr int kBarVFull = 2 * kKSlots;
+    static constexpr int kBarVEmpty = 2 * kKSlots + kVSlots;
+    static constexpr int kBarQFull = 2 * kKSlots + 2 * kVSlots;  // + Q buffer
+    static constexpr int kBarQEmpty = kBarQFull + 2;
+    static constexpr int kBarSFull = kBarQEmpty + 2;   // + S buffer
+    static constexpr int kBarPFull = kBarSFull + 2;    // + P buffer
+    static constexpr int kBarPVDone = kBarPFull + 2;   // + P buffer: PV of that buffer's tile complete
+    static constexpr int kBarDrain = kBarPVDone + 2;
+    static constexpr int kBarNever = kBarDrain + 1;
+    static constexpr int kNumBars = kBarNever + 1;
+    static constexpr int kMiscOff = kBarOff + kNumBars * 8;  // TMEM base address, abort flag
+    static constexpr int kSmemBytes = kMiscOff + 16 + 1024;  // + slack for 1024-byte alignment
+    static constexpr uint32_t kTmemCols = 128;
+    static constexpr uint32_t kColS = 0;  // + 32 * S buffer
+    static constexpr uint32_t kColO = 64;
+    // S^T = K . Q^T: A = K tile (K-major), B = Q^T rows (K-major).
+    static constexpr uint32_t kIdescS = ptx::idesc_bf16_f32_ab(kTile, NC, false, false);
+    // O^T = V^T . P^T: A = V tile read channel-major (MN-major), B = P^T rows (K-major).
+    static constexpr uint32_t kIdescPV = ptx::idesc_bf16_f32_ab(D, NC, true, false);
+};
+static_assert(DCfg::kSmemBytes <= 232448, "decode kernel shared memory");
+static_assert(DCfg::kKOff % 1024 == 0 && DCfg::kVOff % 1024 == 0 && DCfg::kPOff % 1024 == 0,
+              "128-byte swizzled operands need 1024-byte alignment");
+
+struct DParams {
+    const DecUnit* units;
+    const int32_t* cta_off;
+    uint16_t* o;
+    float* lse;
+    int32_t Hq, G, g_shift;  // G = 1 << g_shift
+    float scale_log2;         // softmax scale * log2(e)
+    int32_t* counters;
+    float* part_o;
+    float* part_lse;
+    int32_t* status;
+    uint32_t flags;
+};
+
+__device__ __forceinline__ void dec_producer(const CUtensorMap* tmQ, const CUtensorMap* tmK, const CUtensorMap* tmV,
+                                             const DParams& p, int ubeg, int uend, uint32_t sQ, uint32_t sK,
+                                             uint32_t sV, uint32_t sBar, volatile int32_t* abort_flag) {
+    using C = DCfg;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    const uint64_t once = ptx::policy_evict_first();  // every K/V byte is read once
+    uint32_t kslot = 0, kpar = 0, vslot = 0, vpar = 0;
+    uint32_t k_issued = 0, v_issued = 0, items = 0;
+    uint32_t q_issued[2] = {0u, 0u};
+    bool aborted = false;
+    for (int ui = ubeg; ui < uend && !aborted; ++ui) {
+        const DecUnit u = p.units[ui];
+        if (u.n_tiles <= 0) continue;
+        const int qb = static_cast<int>(items & 1u);
+        if (!bounded_wait(bar(C::kBarQEmpty + qb), (q_issued[qb] & 1u) ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
+            aborted = true;
+            break;
+        }
+        ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + qb), C::kQBytes);
+#pragma unroll
+        for (int b = 0; b < 2; ++b)
+            ptx::tma_load_3d(sQ + qb * C::kQBytes + b * (NC * 128), tmQ, bar(C::kBarQFull + qb), b * 64,
+                             u.kvh * p.G, u.q_tok0);
+        ++q_issued[qb];
+        ++items;
+        for (int j = 0; j < u.n_tiles && !aborted; ++j) {
+            const int row = u.k_row0 + (u.tile0 + j) * kTile;
+            if (!bounded_wait(bar(C::kBarKEmpty + kslot), kpar ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
+                aborted = true;
+                break;
+            }
+            ptx::mbar_arrive_expect_tx(bar(C::kBarKFull + kslot), C::kSlotBytes);
+#pragma unroll
+            for (int b = 0; b < 2; ++b)
+                ptx::tma_load_3d_hint(sK + kslot * C::kSlotBytes + b * (kTile * 128), tmK, bar(C::kBarKFull + kslot),
+                                      b * 64, u.kvh, row, once);
+            ++k_issued;
+            if (++kslot == C::kKSlots) { kslot = 0; kpar ^= 1u; }
+            if (!bounded_wait(bar(C::kBarVEmpty + vslot), vpar ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
+                aborted = true;
+                break;
+            }
+            ptx::mbar_arrive_expect_tx(bar(C::kBarVFull + vslot), C::kSlotBytes);
+#pragma unroll
+            for (int b = 0; b < 2; ++b)
+                ptx::tma_load_3d_hint(sV + vslot * C::kSlotBytes + b * (kTile * 128), tmV, bar(C::kBarVFull + vslot),
+                                      b * 64, u.kvh, row, once);
+            ++v_issued;
+            if (++vslot == C::kVSlots) { vslot = 0; vpar ^= 1u; }
+        }
+    }
+    if (aborted) {
+        // Let every copy still in flight land before the CTA exits: at most
+        // one outstanding load per slot and per Q buffer (the latest).
+        for (uint32_t s = 0; s < static_cast<uint32_t>(C::kKSlots); ++s)
+            if (k_issued > s) {
+                const uint32_t uses = (k_issued - s + C::kKSlots - 1) / C::kKSlots;
+                drain_wait(bar(C::kBarKFull + s), (uses - 1u) & 1u, kDrainLimitNs);
+            }
+        for (uint32_t s = 0; s < static_cast<uint32_t>(C::kVSlots); ++s)
+            if (v_issued > s) {
+                const uint32_t uses = (v_issued - s + C::kVSlots - 1) / C::kVSlots;
+                drain_wait(bar(C::kBarVFull + s), (uses - 1u) & 1u, kDrainLimitNs);
+            }
+        for (int i = 0; i < 2; ++i)
+            if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
+    }
+}
+
+__device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sQ,
+                                        uint32_t sK, uint32_t sV, uint32_t sP, uint32_t sBar,
+                                        volatile int32_t* abort_flag) {
+    using C = DCfg;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    auto wait = [&](int b, uint32_t parity) {
+        return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
+    };
+    uint32_t kslot = 0, kpar = 0, vslot = 0, vpar = 0, items = 0, g = 0;
+    uint32_t q_uses[2] = {0u, 0u};
+    bool ok = true;
+    if (p.flags & kFlagForceTimeout)
+        ok = __all_sync(0xFFFFFFFFu, bounded_wait(bar(C::kBarNever), 0u, abort_flag, p.status, kForcedLimitNs));
+
+    for (int ui = ubeg; ui < uend && ok; ++ui) {
+        const DecUnit u = p.units[ui];
+        const int n = u.n_tiles;
+        if (n <= 0) continue;
+        const int qb = static_cast<int>(items & 1u);
+        if (!(ok = wait(C::kBarQFull + qb, q_uses[qb] & 1u))) break;
+        ++q_uses[qb];
+        ++items;
+        const uint32_t qaddr = sQ + qb * C::kQBytes;
+        // S(gg) = K . Q^T from the next K slot into S buffer gg & 1.
+        auto issue_s = [&](uint32_t gg) -> bool {
+            if (!wait(C::kBarKFull + kslot, kpar)) return false;
+            ptx::tc_fence_after();
+            const uint32_t kaddr = sK + kslot * C::kSlotBytes;
+#pragma unroll
+            for (int ks = 0; ks < D / 16; ++ks) {
+                const uint32_t aoff = (ks >> 2) * (kTile * 128) + (ks & 3) * 32;
+                const uint32_t boff = (ks >> 2) * (NC * 128) + (ks & 3) * 32;
+                ptx::mma_ss_warp(tmem + C::kColS + 32u * (gg & 1u), ptx::sdesc_sw128(kaddr + aoff, 16, 1024),
+                                 ptx::sdesc_sw128(qaddr + boff, 16, 1024), C::kIdescS, ks > 0 ? 1u : 0u);
+            }
+            ptx::tc_commit_warp(bar(C::kBarSFull + static_cast<int>(gg & 1u)));
+            ptx::tc_commit_warp(bar(C::kBarKEmpty + kslot));
+            if (++kslot == C::kKSlots) { kslot = 0; kpar ^= 1u; }
+            return true;
+        };
+        if (!(ok = issue_s(g))) break;
+        if (n > 1 && !(ok = issue_s(g + 1))) break;
+        if (n <= 2) ptx::tc_commit_warp(bar(C::kBarQEmpty + qb));
+        for (int j = 0; j < n; ++j) {
+            const uint32_t gj = g + static_cast<uint32_t>(j);
+            const int pb = static_cast<int>(gj & 1u);
+            if (!(ok = wait(C::kBarPFull + pb, (gj >> 1) & 1u))) break;
+            if (!(ok = wait(C::kBarVFull + vslot, vpar))) break;
+            ptx::tc_fence_after();
+            const uint32_t vaddr = sV + vslot * C::kSlotBytes;
+            const uint32_t paddr = sP + pb * C::kPBytes;
+#pragma unroll
+            for (int ks = 0; ks < kTile / 16; ++ks) {
+                // V tile is [keys][d]: read channel-major, 16 keys per step,
+                // 64-channel blocks kTile * 128 bytes apart, 8-key groups 1024 apart.
+                const uint32_t boff = (ks >> 2) * (NC * 128) + (ks & 3) * 32;
+                ptx::mma_ss_warp(tmem + C::kColO, ptx::sdesc_sw128(vaddr + ks * (16 * 128), kTile * 128, 1024),
+                                 ptx::sdesc_sw128(paddr + boff, 16, 1024), C::kIdescPV,
+                                 (j > 0 || ks > 0) ? 1u : 0u);
+            }
+            ptx::tc_commit_warp(bar(C::kBarPVDone + pb));
+            ptx::tc_commit_warp(bar(C::kBarVEmpty + vslot));
+            if (++vslot == C::kVSlots) { vslot = 0; vpar ^= 1u; }
+            if (j + 2 < n) {
+                if (!(ok = issue_s(gj + 2))) break;
+                if (j + 3 == n) ptx::tc_commit_warp(bar(C::kBarQEmpty + qb));
+            }
+        }
+        g += static_cast<uint32_t>(n);
+    }
+    // Every MMA this warp issued must finish before TMEM is released.
+    ptx::tc_commit_warp(bar(C::kBarDrain));
+    drain_wait(bar(C::kBarDrain), 0u, kDrainLimitNs);
+}
+
+// Reduces v[c] over the 128 threads of the softmax warpgroup for each of the
+// NCOL columns and gives every thread all NCOL results.  Within a warp, lanes
+// 8, 16, ... apart are first combined column by column until NCOL lanes are
+// left per column; the columns are then halved with butterfly exchanges, so
+// lane l ends with column l mod NCOL.  The four warps combine through shared
+// memory.
+template <int NCOL, bool kMax>
+__device__ __forceinline__ void wg_reduce(const float* v, float* out, float* red, int warp, int lane) {
+    float x[NCOL];
+#pragma unroll
+    for (int c = 0; c < NCOL; ++c) x[c] = v[c];
+#pragma unroll
+    for (int o = 16; o >= NCOL; o >>= 1) {
+#pragma unroll
+        for (int c = 0; c < NCOL; ++c) {
+            const float y = __shfl_xor_sync(0xFFFFFFFFu, x[c], o);
+            x[c] = kMax ? fmaxf(x[c], y) : x[c] + y;
+        }
+    }
+#pragma unroll
+    for (int o = NCOL / 2; o >= 1; o >>= 1) {  // o = number of columns kept
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float send = upper ? x[i] : x[i + o];
+            const float keep = upper ? x[i + o] : x[i];
+            const float recv = __shfl_xor_sync(0xFFFFFFFFu, send, o);
+            x[i] = kMax ? fmaxf(keep, recv) : keep + recv;
+        }
+    }
+    red[warp * 32 + lane] = x[0];
+    ptx::bar_sync(kBarWG, kWGThreads);
+    float t = red[lane];
+#pragma unroll
+    for (int w = 1; w < 4; ++w) t = kMax ? fmaxf(t, red[w * 32 + lane]) : t + red[w * 32 + lane];
+#pragma unroll
+    for (int c = 0; c < NCOL; ++c) out[c] = __shfl_sync(0xFFFFFFFFu, t, c);
+}
+
+__device__ __forceinline__ uint16_t f32_to_bf16_bits(float x) {
+    return static_cast<uint16_t>(ptx::pack_bf16x2(x, 0.f) & 0xFFFFu);
+}
+
+__device__ __forceinline__ int64_t out_row(const DParams& p, const DecUnit& u, int c) {
+    return static_cast<int64_t>(u.q_tok0 + (c >> p.g_shift)) * p.Hq + u.kvh * p.G + (c & (p.G - 1));
+}
+
+// Softmax warpgroup.  NCOL (8, 16 or 32) is the number of S^T / O^T columns
+// it processes: the largest G * Lq of the batch rounded up.  Columns beyond
+// a unit's own G * Lq are masked and never written to P^T (zero there).
+template <int NCOL>
+__device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sP,
+                                            float* sRed, uint32_t sBar, int tid, volatile int32_t* abort_flag) {
+    using C = DCfg;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    const int warp = tid >> 5, lane = tid & 31;
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const uint32_t tS = tmem + lane_off + C::kColS;
+    const uint32_t tO = tmem + lane_off + C::kColO;
+    const float cl = p.scale_log2;
+    const int gs = p.g_shift;
+    // P^T element (column c, key tid): 64-key block, row c, 16-byte chunk swizzled by c mod 8.
+    const uint32_t p_thread = static_cast<uint32_t>((tid >> 6) * (NC * 128) + ((tid & 7) << 1));
+    const uint32_t p_chunk = static_cast<uint32_t>((tid & 63) >> 3);
+    uint32_t g = 0;
+    int red_buf = 0;
+    auto red_ptr = [&]() {
+        float* r = sRed + red_buf * 128;
+        red_buf ^= 1;
+        return r;
+    };
+    auto warp_wait = [&](int b, uint32_t parity) {
+        return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
+    };
+    // A wait's outcome is made uniform over the warpgroup before anyone acts
+    // on it, so no warp leaves while the others sit in a named barrier.
+    auto wg_wait = [&](int b, uint32_t parity) { return ptx::bar_red_and(kBarWG, kWGThreads, warp_wait(b, parity)); };
+
+    for (int ui = ubeg; ui < uend; ++ui) {
+        const DecUnit u = p.units[ui];
+        const int ncols = u.nq << gs;
+        if (u.n_tiles <= 0) {  // the sequence has no key: O = 0, LSE = -inf
+#pragma unroll
+            for (int c = 0; c < NCOL; ++c) {
+                if (c >= ncols) break;
+                const int64_t row = out_row(p, u, c);
+                p.o[row * D + tid] = 0;
+                if (tid == c) p.lse[row] = -INFINITY;
+            }
+            continue;
+        }
+        const int lim0 = u.Lk - u.nq;  // column c sees keys 0 .. lim0 + c / G
+        float base[NCOL], l[NCOL], lh[NCOL];
+#pragma unroll
+        for (int c = 0; c < NCOL; ++c) {
+            base[c] = -INFINITY;
+            l[c] = 0.f;
+            lh[c] = 0.f;
+        }
+        for (int j = 0; j < u.n_tiles; ++j) {
+            const uint32_t b = g & 1u;
+            // S(g) ready, and P buffer b free (last read by PV(g - 2)).
+            bool ok = warp_wait(C::kBarSFull + static_cast<int>(b), (g >> 1) & 1u);
+            if (ok && g >= 2u) ok = warp_wait(C::kBarPVDone + static_cast<int>(b), ((g - 2u) >> 1) & 1u);
+            float s[NCOL];
+            bool need = j == 0;
+            if (ok) {
+                ptx::tc_fence_after();
+                uint32_t sr[NCOL];
+                ptx::tmem_ld_n<NCOL>(tS + 32u * b, sr);
+                ptx::tmem_wait_ld();
+                ptx::tmem_ld_fence<NCOL>(sr);
+                const int key = (u.tile0 + j) * kTile + tid;
+#pragma unroll
+                for (int c = 0; c < NCOL; ++c) {
+                    const bool vis = c < ncols && key <= lim0 + (c >> gs);
+                    s[c] = vis ? __uint_as_float(sr[c]) * cl : -INFINITY;
+                    need |= s[c] - base[c] > kRebaseSlack;
+                }
+            }
+            // One warpgroup barrier per tile in the common case: it carries
+            // both "some column needs a new base" and "some wait failed".
+            if (ptx::bar_red_or(kBarWG, kWGThreads, need || !ok)) {
+                if (!ptx::bar_red_and(kBarWG, kWGThreads, ok)) return;
+                float tmax[NCOL];
+                wg_reduce<NCOL, true>(s, tmax, red_ptr(), warp, lane);
+                bool scaled = false;
+                float alpha[NCOL];
+#pragma unroll
+                for (int c = 0; c < NCOL; ++c) {
+                    const float nb = fmaxf(base[c], tmax[c]);
+                    alpha[c] = nb == base[c] ? 1.f : (base[c] == -INFINITY ? 0.f : ptx::ex2_approx(base[c] - nb));
+                    base[c] = nb;
+                    l[c] *= alpha[c];
+                    lh[c] *= alpha[c];
+                    scaled |= alpha[c] != 1.f;
+                }
+                // base and tmax are the same in every thread, so is `scaled`.
+                if (j > 0 && scaled) {
+                    // O holds PV of the earlier tiles on the old bases; the
+                    // latest of them, PV(g - 1), must be complete.
+                    const uint32_t gp = g - 1u;
+                    if (!wg_wait(C::kBarPVDone + static_cast<int>(gp & 1u), (gp >> 1) & 1u)) return;
+                    ptx::tc_fence_after();
+                    uint32_t ov[NCOL];
+                    ptx::tmem_ld_n<NCOL>(tO, ov);
+                    ptx::tmem_wait_ld();
+                    ptx::tmem_ld_fence<NCOL>(ov);
+#pragma unroll
+                    for (int c = 0; c < NCOL; ++c) ov[c] = __float_as_uint(__uint_as_float(ov[c]) * alpha[c]);
+                    ptx::tmem_st_n<NCOL>(tO, ov);
+                    ptx::tmem_wait_st();
+                }
+            }
+            const uint32_t pbase = sP + b * C::kPBytes + p_thread;
+#pragma unroll
+            for (int c = 0; c < NCOL; ++c) {
+                const float pv = ptx::ex2_approx(s[c] - (base[c] == -INFINITY ? 0.f : base[c]));
+                const uint32_t pk = ptx::pack_bf16x2(pv, 0.f);
+                l[c] += pv;
+                lh[c] += ptx::bf16lo_to_f32(pk);
+                if (c < ncols) ptx::st_shared_u16(pbase + c * 128 + ((p_chunk ^ (c & 7)) << 4), static_cast<uint16_t>(pk));
+            }
+            ptx::fence_proxy_async_smem();
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(bar(C::kBarPFull + static_cast<int>(b)));
+            ++g;
+        }
+        // epilogue: wait for the unit's last PV
+        const uint32_t gl = g - 1u;
+        if (!wg_wait(C::kBarPVDone + static_cast<int>(gl & 1u), (gl >> 1) & 1u)) return;
+        ptx::tc_fence_after();
+        uint32_t ov[NCOL];
+        ptx::tmem_ld_n<NCOL>(tO, ov);
+        ptx::tmem_wait_ld();
+        ptx::tmem_ld_fence<NCOL>(ov);
+        float L[NCOL], LH[NCOL];
+        wg_reduce<NCOL, false>(l, L, red_ptr(), warp, lane);
+        wg_reduce<NCOL, false>(lh, LH, red_ptr(), warp, lane);
+        if (u.part < 0) {
+            // O is normalised by the sum of the rounded weights the PV MMA
+            // used (a weighted mean of V rows); LSE uses the unrounded sum.
+#pragma unroll
+            for (int c = 0; c < NCOL; ++c) {
+                if (c >= ncols) break;
+                const int64_t row = out_row(p, u, c);
+                const float inv = LH[c] > 0.f ? 1.f / LH[c] : 0.f;
+                p.o[row * D + tid] = f32_to_bf16_bits(__uint_as_float(ov[c]) * inv);
+                if (tid == c) p.lse[row] = L[c] > 0.f ? (base[c] + log2f(L[c])) * kLn2Dec : -INFINITY;
+            }
+            continue;
+        }
+        // split key range: partial (normalised O, log2-domain LSE)
+        float* po = p.part_o + static_cast<int64_t>(u.part) * NC * D;
+#pragma unroll
+        for (int c = 0; c < NCOL; ++c) {
+            if (c >= ncols) break;
+            po[c * D + tid] = LH[c] > 0.f ? __uint_as_float(ov[c]) / LH[c] : 0.f;
+            if (tid == c) p.part_lse[u.part * NC + c] = L[c] > 0.f ? base[c] + log2f(L[c]) : -INFINITY;
+        }
+        __threadfence();
+        ptx::bar_sync(kBarWG, kWGThreads);
+        bool last = false;
+        if (tid == 0) last = atomicAdd(p.counters + u.group, 1) == u.n_chunks - 1;
+        last = ptx::bar_red_or(kBarWG, kWGThreads, last);
+        if (!last) continue;
+        // This unit finished last: merge the (sequence, kv head)'s partials,
+        // O = sum_k 2^(lse_k - lse) O_k with lse = log2 sum_k 2^lse_k.
+        __threadfence();
+        const int part0 = u.part - u.chunk;
+        for (int c = 0; c < ncols; ++c) {
+            float m = -INFINITY;
+            for (int k = 0; k < u.n_chunks; ++k) m = fmaxf(m, __ldcg(p.part_lse + (part0 + k) * NC + c));
+            float acc = 0.f, wsum = 0.f;
+            if (m != -INFINITY) {
+                for (int k = 0; k < u.n_chunks; ++k) {
+                    const float w = ptx::ex2_approx(__ldcg(p.part_lse + (part0 + k) * NC + c) - m);
+                    wsum += w;
+                    acc += w * __ldcg(p.part_o + (static_cast<int64_t>(part0 + k) * NC + c) * D + tid);
+                }
+            }
+            const int64_t row = out_row(p, u, c);
+            p.o[row * D + tid] = f32_to_bf16_bits(wsum > 0.f ? acc / wsum : 0.f);
+            if (tid == 0) p.lse[row] = wsum > 0.f ? (m + log2f(wsum)) * kLn2Dec : -INFINITY;
+        }
+    }
+}
+
+template <int NCOL>
+__global__ void __launch_bounds__(kThreadsDec, 1)
+    opattn_decode_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                         const __grid_constant__ CUtensorMap tmV, const DParams p) {
+    using C = DCfg;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    const uint32_t raw = ptx::smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* gbase = smem_raw + (base - raw);
+    const uint32_t sQ = base + C::kQOff;
+    const uint32_t sK = base + C::kKOff;
+    const uint32_t sV = base + C::kVOff;
+    const uint32_t sP = base + C::kPOff;
+    const uint32_t sBar = base + C::kBarOff;
+    float* sRed = reinterpret_cast<float*>(gbase + C::kRedOff);
+    volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(gbase + C::kMiscOff);
+    volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(gbase + C::kMiscOff + 4);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5;
+    const int lane = tid & 31;
+
+    if (tid == 0) {
+        for (int i = 0; i < C::kKSlots; ++i) {
+            ptx::mbar_init(sBar + 8u * (C::kBarKFull + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarKEmpty + i), 1);
+        }
+        for (int i = 0; i < C::kVSlots; ++i) {
+            ptx::mbar_init(sBar + 8u * (C::kBarVFull + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarVEmpty + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(sBar + 8u * (C::kBarQFull + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarQEmpty + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarSFull + i), 1);
+            ptx::mbar_init(sBar + 8u * (C::kBarPFull + i), kWGThreads);
+            ptx::mbar_init(sBar + 8u * (C::kBarPVDone + i), 1);
+        }
+        ptx::mbar_init(sBar + 8u * C::kBarDrain, 1);
+        ptx::mbar_init(sBar + 8u * C::kBarNever, 1);
+        *abort_flag = 0;
+        ptx::fence_mbar_init();
+    }
+    if (tid < static_cast<int>(kWGThreads)) {
+        // Columns a unit does not use are never written: start them finite.
+        const uint32_t dst = sP + static_cast<uint32_t>(tid) * (2 * C::kPBytes / kWGThreads);
+#pragma unroll
+        for (int i = 0; i < 2 * C::kPBytes / static_cast<int>(kWGThreads); i += 16) ptx::st_shared_v4(dst + i, 0u, 0u, 0u, 0u);
+        ptx::fence_proxy_async_smem();
+    }
+    if (warp == kWarpMmaDec) {
+        ptx::tmem_alloc(ptx::smem_addr(const_cast<uint32_t*>(tmem_slot)), C::kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == kWarpProducerDec && lane == 0) {
+        ptx::prefetch_tmap(&tmQ);
+        ptx::prefetch_tmap(&tmK);
+        ptx::prefetch_tmap(&tmV);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int ubeg = p.cta_off[blockIdx.x];
+    const int uend = p.cta_off[blockIdx.x + 1];
+
+    if (warp < 4) {
+        dec_softmax<NCOL>(p, ubeg, uend, tmem, sP, sRed, sBar, tid, abort_flag);
+    } else if (warp == kWarpProducerDec) {
+        if (lane == 0) dec_producer(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sK, sV, sBar, abort_flag);
+        __syncwarp();
+    } else if (warp == kWarpMmaDec) {
+        dec_mma(p, ubeg, uend, tmem, sQ, sK, sV, sP, sBar, abort_flag);
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == kWarpMmaDec) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+template <int NCOL>
+int launch_ncol(const DecodeLaunchArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                const DParams& kp, cudaStream_t stream) {
+    using C = DCfg;
+    static std::mutex mu;
+    static bool attr_done[128] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        if (dev < 0 || dev >= 128 || !attr_done[dev]) {
+            e = cudaFuncSetAttribute(opattn_decode_kernel<NCOL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     C::kSmemBytes);
+            if (e != cudaSuccess) return e;
+            if (dev >= 0 && dev < 128) attr_done[dev] = true;
+        }
+    }
+    opattn_decode_kernel<NCOL><<<a.n_cta, kThreadsDec, C::kSmemBytes, stream>>>(tq, tk, tv, kp);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return -1;
+    const int G = a.Hq / a.Hkv;
+    if (G <= 0 || NC % G != 0 || a.max_cols <= 0 || a.max_cols > NC) return -5;
+    int g_shift = 0;
+    while ((1 << g_shift) < G) ++g_shift;
+    CUtensorMap tq, tk, tv;
+    const void* kb = a.total_k > 0 ? a.k : a.q;
+    const void* vb = a.total_k > 0 ? a.v : a.q;
+    const uint64_t krows = a.total_k > 0 ? static_cast<uint64_t>(a.total_k) : 1;
+    if (!encode_3d(fn, &tq, a.q, D, a.Hq, a.total_q, G, NC / G)) return -2;
+    if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, kTile)) return -3;
+    if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, kTile)) return -4;
+    DParams kp;
+    kp.units = a.units;
+    kp.cta_off = a.cta_off;
+    kp.o = static_cast<uint16_t*>(a.o);
+    kp.lse = a.lse;
+    kp.Hq = a.Hq;
+    kp.G = G;
+    kp.g_shift = g_shift;
+    kp.scale_log2 = a.scale * kLog2eDec;
+    kp.counters = a.counters;
+    kp.part_o = a.part_o;
+    kp.part_lse = a.part_lse;
+    kp.status = a.status;
+    kp.flags = a.flags;
+    if (a.max_cols <= 8) return launch_ncol<8>(a, tq, tk, tv, kp, stream);
+    if (a.max_cols <= 16) return launch_ncol<16>(a, tq, tk, tv, kp, stream);
+    return launch_ncol<32>(a, tq, tk, tv, kp, stream);
+}
+
+}  // namespace opattn

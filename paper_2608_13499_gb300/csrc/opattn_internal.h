@@ -65,9 +65,59 @@ constexpr int32_t kNoAllocMaxCtas = 1024;
 // cudaError_t as int.
 int noalloc_scratch(void** ptr, size_t* bytes);
 
+// ------------------------------------------------------------------ decode
+// The decode kernel (opattn_decode.cu) computes the same attention for
+// sequences with few query tokens: the G * Lq (query token, head) pairs of
+// one kv head form the N = kDecCols columns of transposed score and output
+// tiles, the 128 keys of a key tile (or the 128 channels of d) their rows.
+// Long key ranges are cut into chunks that run as separate work units; each
+// writes a partial (O, LSE) and the last unit of a (sequence, kv head) to
+// finish merges them.
+constexpr int kDecCols = 32;
+constexpr int kDecHeadDim = 128;
+
+struct DecUnit {
+    int32_t q_tok0;    // packed query row of the sequence's first token
+    int32_t nq;        // query tokens of the sequence (nq * G <= kDecCols)
+    int32_t k_row0;    // packed key row of the sequence's first key
+    int32_t Lk;        // keys in the sequence
+    int32_t kvh;       // kv head
+    int32_t tile0;     // first key tile of the chunk
+    int32_t n_tiles;   // key tiles of the chunk (0: the sequence has no key)
+    int32_t part;      // partial slot of the chunk, -1 when the chunk is the whole sequence
+    int32_t group;     // merge counter of the (sequence, kv head), -1 when not split
+    int32_t chunk;     // chunk index within the (sequence, kv head)
+    int32_t n_chunks;  // chunks of the (sequence, kv head)
+    int32_t seq;       // sequence index (diagnostics only)
+};
+static_assert(sizeof(DecUnit) == 48, "DecUnit must stay 48 bytes");
+
+struct DecodeLaunchArgs {
+    const void* q;
+    const void* k;
+    const void* v;
+    void* o;
+    float* lse;
+    int64_t total_q;
+    int64_t total_k;
+    int32_t Hq, Hkv;
+    float scale;
+    const DecUnit* units;     // device
+    const int32_t* cta_off;   // device, n_cta + 1
+    int32_t n_cta;
+    int32_t max_cols;         // largest G * Lq of the batch (<= kDecCols)
+    int32_t* counters;        // device, one per split (sequence, kv head), zero at launch
+    float* part_o;            // device, [parts][kDecCols][kDecHeadDim]
+    float* part_lse;          // device, [parts][kDecCols] (log2 domain)
+    int32_t* status;          // device
+    uint32_t flags;
+};
+
 // Implemented in opattn_kernel.cu.  Returns a cudaError_t (as int) or a
 // negative value when the tensor maps cannot be encoded.
 int launch_prefill(const LaunchArgs& a, cudaStream_t stream);
+// Implemented in opattn_decode.cu; same return convention.
+int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream);
 // Shared memory bytes the kernel needs for head dim d (0 if unsupported).
 int kernel_smem_bytes(int d);
 

@@ -33,6 +33,7 @@
 #include <cstdint>
 #include <mutex>
 
+#include "device_common.cuh"
 #include "opattn_internal.h"
 #include "ptx.cuh"
 
@@ -44,9 +45,6 @@ constexpr int kWarpProducer = 0;
 constexpr int kWarpMma = 1;
 constexpr int kWarpSoftmax = 4;  // first softmax warp; warps 4..7 -> M-tile 0, 8..11 -> M-tile 1
 
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: no legitimate wait comes close
-constexpr uint64_t kForcedLimitNs = 20000000ull;  // 20 ms: the forced-timeout test
-constexpr uint64_t kDrainLimitNs = 200000000ull;  // in-flight copies / MMAs after an abort
 // Largest sum of one tile's exponentials accepted with a reused subtraction
 // base; fp32 sums and the fp32 O accumulator stay far from overflow.
 constexpr float kMaxTileSum = 18446744073709551616.0f;  // 2^64
@@ -103,33 +101,6 @@ struct KParams {
     int32_t* status;
     uint32_t flags;
 };
-
-// Wait for the phase of parity `parity` of `bar`.  Gives up when another
-// thread of the CTA has aborted, or after `limit_ns`, in which case it
-// raises the CTA abort flag and records a timeout in the status word.
-__device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, volatile int32_t* abort_flag,
-                                             int32_t* status, uint64_t limit_ns) {
-    if (ptx::mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = ptx::globaltimer_ns();
-    for (;;) {
-        if (ptx::mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (ptx::globaltimer_ns() - t0 > limit_ns) {
-            *abort_flag = 1;
-            atomicCAS(status, kDevOk, kDevTimeout);
-            return false;
-        }
-    }
-}
-
-// Wait used while shutting down after an abort: ignores the abort flag and
-// returns silently after `limit_ns`.
-__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
-    const uint64_t t0 = ptx::globaltimer_ns();
-    while (!ptx::mbar_try_wait(bar, parity)) {
-        if (ptx::globaltimer_ns() - t0 > limit_ns) return;
-    }
-}
 
 template <int D>
 __device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUtensorMap* tmK,
@@ -571,39 +542,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// ------------------------------------------------------------------- host
-
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void* ptr = nullptr;
-        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    });
-    return fn;
-}
-
-// [rows, heads, d] bf16 tensor, box of (64 channels, box_heads, box_rows),
-// 128-byte swizzle; out-of-range rows read as zero.
-bool encode_3d(EncodeTiledFn fn, CUtensorMap* map, const void* base, uint64_t d, uint64_t heads, uint64_t rows,
-               uint32_t box_heads, uint32_t box_rows) {
-    const cuuint64_t dims[3] = {d, heads, rows};
-    const cuuint64_t strides[2] = {d * 2, heads * d * 2};
-    const cuuint32_t box[3] = {64, box_heads, box_rows};
-    const cuuint32_t estr[3] = {1, 1, 1};
-    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int D>
 int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     using C = Cfg<D>;
@@ -662,6 +600,35 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
 }
 
 }  // namespace
+
+// ------------------------------------------------------------------- host
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+// [rows, heads, d] bf16 tensor, box of (64 channels, box_heads, box_rows),
+// 128-byte swizzle; out-of-range rows read as zero.
+bool encode_3d(EncodeTiledFn fn, CUtensorMap* map, const void* base, uint64_t d, uint64_t heads, uint64_t rows,
+               uint32_t box_heads, uint32_t box_rows) {
+    const cuuint64_t dims[3] = {d, heads, rows};
+    const cuuint64_t strides[2] = {d * 2, heads * d * 2};
+    const cuuint32_t box[3] = {64, box_heads, box_rows};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 int launch_prefill(const LaunchArgs& a, cudaStream_t stream) {
     if (a.d == 64) return launch_d<64>(a, stream);

@@ -344,7 +344,7 @@ def profile_accuracy(n_train: int, n_test: int, seed: int = 0, key: OperatorKey 
     integer = [True, True] + ([False] if s_range else [])
     train = sample_points(n_train, rng, ranges, integer)
     test = sample_points(n_test, rng, ranges, integer, corners=False, stratified=False)
-    buf = _Buffers(int(b_range[1] * l_range[1]), key.Hq, key.Hkv, key.d)
+    buf = _Buffers(int(b_range[1] * l_range[1]), *key.shape)
     sms = n_sms()
 
     def run(p):

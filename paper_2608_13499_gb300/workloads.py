@@ -208,5 +208,25 @@ def chunked(seed: int = 0) -> Workload:
                     32, 8, 128, 1.0, seed)
 
 
+def decode_llama3_70b(seed: int = 0) -> Workload:
+    """64 requests decoding one token each over 8192 cached keys; Hq 64, Hkv 8, d 128."""
+    return Workload("decode_llama3_70b_64x8192", [1] * 64, [8192] * 64, 64, 8, 128, 1.0, seed)
+
+
+def decode_llama3_8b(seed: int = 0) -> Workload:
+    """128 requests decoding one token each over lognormal(median 4096, sigma 0.8) in [16, 32768]
+    cached keys; Hq 32, Hkv 8, d 128."""
+    lens = lognormal_lengths(seed, 128, median=4096.0, sigma=0.8, lo=16, hi=32768)
+    return Workload("decode_llama3_8b_ragged_128seq", [1] * 128, lens, 32, 8, 128, 1.0, seed)
+
+
+def decode_spec4_llama3_70b(seed: int = 0) -> Workload:
+    """32 requests verifying 4 speculative tokens each over 16384 cached keys; Hq 64, Hkv 8, d 128."""
+    return Workload("decode_spec4_llama3_70b_32x16384", [4] * 32, [16384] * 32, 64, 8, 128, 1.0, seed)
+
+
+DECODE = {"decode_llama3_70b": decode_llama3_70b, "decode_llama3_8b": decode_llama3_8b,
+          "decode_spec4_llama3_70b": decode_spec4_llama3_70b}
+
 STANDARD = {"tiny": tiny, "llama3_8b": llama3_8b, "llama3_70b": llama3_70b,
             "bursty": bursty, "chunked": chunked}

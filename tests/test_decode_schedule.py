@@ -1,0 +1,135 @@
+"""Decode scheduler and argument checks of the decode entry points (no GPU).
+
+Checked against brute-force enumeration: every (sequence, kv head, key tile)
+is covered by exactly one chunk, chunks of a pair are contiguous, equal to
+within one tile and numbered in order, partial slots and merge groups are
+unique and dense, and the assignment obeys the longest-first rule.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+import paper_2608_13499_gb300 as pkg
+from paper_2608_13499_gb300 import build as pbuild
+
+BN = 128
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    pbuild.build()
+    return pkg.load()
+
+
+def table(units):
+    return {name: units[:, i] for i, name in enumerate(pkg.DEC_UNIT_FIELDS)}
+
+
+CASES = [
+    # (q_lens, k_lens, Hq, Hkv, n_cta)
+    ([1] * 9, [1, 2, 127, 128, 129, 255, 257, 1000, 3000], 16, 2, 152),
+    ([2, 2, 2, 2], [5, 130, 700, 2049], 32, 8, 152),
+    ([4, 4, 4, 4], [4, 64, 513, 4100], 16, 2, 7),
+    ([3, 1, 0, 2], [1, 0, 5, 2], 16, 2, 152),            # Lq > Lk, no keys, no queries
+    ([1, 1], [32768, 32768], 64, 8, 152),                 # long contexts are split
+    ([1] * 64, [8192] * 64, 64, 8, 152),
+    ([1], [40000], 8, 1, 1),                              # one CTA still splits into ~6 chunks
+    ([1] * 5, [300, 9000, 17, 128 * 40, 1], 32, 1, 152),  # G = 32
+]
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_chunks_cover_every_key_tile_once(case):
+    lq, lk, Hq, Hkv, n_cta = case
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_decode_schedule(cu_q, cu_k, Hq, Hkv, 128, n_cta)
+    t = table(units)
+    seen = {}
+    for i in range(len(units)):
+        s, h = int(t["seq"][i]), int(t["kvh"][i])
+        assert lq[s] > 0
+        assert t["q_tok0"][i] == cu_q[s] and t["nq"][i] == lq[s]
+        assert t["k_row0"][i] == cu_k[s] and t["Lk"][i] == lk[s]
+        seen.setdefault((s, h), []).append(i)
+    want_pairs = {(s, h) for s in range(len(lq)) if lq[s] > 0 for h in range(Hkv)}
+    assert set(seen) == want_pairs
+    parts, groups = [], []
+    for (s, h), idx in seen.items():
+        n_t = (lk[s] + BN - 1) // BN
+        idx = sorted(idx, key=lambda i: t["chunk"][i])
+        n_chunks = len(idx)
+        assert all(t["n_chunks"][i] == n_chunks for i in idx)
+        assert [int(t["chunk"][i]) for i in idx] == list(range(n_chunks))
+        covered = []
+        for i in idx:
+            covered += list(range(t["tile0"][i], t["tile0"][i] + t["n_tiles"][i]))
+        assert covered == list(range(n_t))                   # contiguous, in order, exactly once
+        sizes = [int(t["n_tiles"][i]) for i in idx]
+        assert max(sizes) - min(sizes) <= 1
+        if n_chunks == 1:
+            assert t["part"][idx[0]] == -1 and t["group"][idx[0]] == -1
+        else:
+            assert min(sizes) >= 2
+            g = {int(t["group"][i]) for i in idx}
+            assert len(g) == 1 and -1 not in g
+            groups.append(g.pop())
+            p0 = int(t["part"][idx[0]])
+            assert [int(t["part"][i]) for i in idx] == list(range(p0, p0 + n_chunks))
+            parts += list(range(p0, p0 + n_chunks))
+    assert sorted(groups) == list(range(len(groups)))
+    assert sorted(parts) == list(range(len(parts)))
+    # longest first within each CTA, CTAs used = min(n_cta, units)
+    assert len(offs) - 1 == min(n_cta, len(units)) and offs[-1] == len(units)
+    cost = t["n_tiles"].astype(np.int64) + 1
+    for c in range(len(offs) - 1):
+        assert np.all(np.diff(cost[offs[c]:offs[c + 1]]) <= 0)
+    loads = np.array([cost[offs[c]:offs[c + 1]].sum() for c in range(len(offs) - 1)])
+    assert loads.max() <= (4.0 / 3.0) * max(cost.sum() / (len(offs) - 1), cost.max()) + 1e-9
+
+
+def test_long_contexts_are_split_for_parallelism():
+    units, _ = pkg.opattn_decode_schedule([0, 1, 2], [0, 32768, 65536], 64, 8, 128, 152)
+    t = table(units)
+    # 2 x 8 pairs of 256 tiles on 152 CTAs: chunks of ceil(27 / 6) = 5 tiles -> 52 chunks per pair
+    assert len(units) == 16 * 52 and set(t["n_chunks"]) == {52}
+    # a short batch is not split
+    units, _ = pkg.opattn_decode_schedule([0, 1, 2], [0, 500, 1000], 64, 8, 128, 152)
+    assert set(table(units)["n_chunks"]) == {1}
+
+
+A = 0x10000
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(d=64), pkg.OPATTN_ERR_UNSUPPORTED),                          # decode kernel is d = 128 only
+    (dict(Hq=6, Hkv=2), pkg.OPATTN_ERR_UNSUPPORTED),                   # G = 3 does not divide 32
+    (dict(Hq=64, Hkv=1), pkg.OPATTN_ERR_UNSUPPORTED),                  # G = 64 > 32 columns
+    (dict(cu_q=(0, 5), cu_k=(0, 9)), pkg.OPATTN_ERR_UNSUPPORTED),      # 5 tokens x G 8 > 32 columns
+    (dict(Hq=6, Hkv=4), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(q=A + 8), pkg.OPATTN_ERR_MISALIGNED),
+    (dict(lse=None), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(scale=0.0), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(cu_q=(0, 0), cu_k=(0, 7)), pkg.OPATTN_OK),                   # no query rows: nothing to do
+])
+def test_decode_argument_errors(kwargs, status):
+    args = dict(q=A, k=A, v=A, o=A, lse=A, cu_q=(0, 1), cu_k=(0, 9), n_seq=1, Hq=16, Hkv=2, d=128, scale=0.125)
+    args.update(kwargs)
+    st = pkg.opattn_decode(args["q"], args["k"], args["v"], args["o"], args["lse"], args["cu_q"], args["cu_k"],
+                           args["n_seq"], args["Hq"], args["Hkv"], args["d"], args["scale"], stream=0, check=False)
+    assert st == status
+
+
+def test_decode_plan_and_schedule_validate():
+    with pytest.raises(pkg.OpattnError) as e:
+        pkg.Plan((0, 1), (0, 9), 16, 2, 64, decode=True)
+    assert e.value.status == pkg.OPATTN_ERR_UNSUPPORTED
+    lib = pkg.load()
+    cu = np.array([0, 1], dtype=np.int32)
+    n_units, n_used = ctypes.c_int64(0), ctypes.c_int32(0)
+    st = lib.opattn_decode_schedule(cu.ctypes.data_as(ctypes.c_void_p), cu.ctypes.data_as(ctypes.c_void_p), 1,
+                                    16, 2, 128, 0, None, 0, None, ctypes.byref(n_units), ctypes.byref(n_used))
+    assert st == pkg.OPATTN_ERR_INVALID_ARG                             # n_ctas must be positive
+    assert pkg.opattn_decode_checked(A, A, A, A, A, (0, 1), (0, 9), 1, 16, 2, 128, 0.1, stream=0,
+                                     flags=0x40) == pkg.OPATTN_ERR_INVALID_ARG
