@@ -429,7 +429,8 @@ void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geome
     out->max_cols = max_cols;
 }
 
-// Device work area: [cta_off | pad 32 | units | counters (n_groups) | status |
+// Device work area: [cta_off | pad 32 | units | counters (2 per group: one per
+// softmax warpgroup) | status |
 // pad 256 | part_lse (n_parts x kDecCols) | part_o (n_parts x kDecCols x d)].
 // The counters and the status word are contiguous and zeroed before every
 // launch.
@@ -440,7 +441,7 @@ DecodeLayout decode_layout(const DecodeSchedule& s) {
     DecodeLayout w;
     w.off_units = (s.cta_off.size() * sizeof(int32_t) + 31) / 32 * 32;
     w.off_counters = w.off_units + s.units.size() * sizeof(DecUnit);
-    w.off_status = w.off_counters + static_cast<size_t>(s.n_groups) * sizeof(int32_t);
+    w.off_status = w.off_counters + 2 * static_cast<size_t>(s.n_groups) * sizeof(int32_t);
     w.upload_bytes = w.off_counters;
     w.zero_bytes = w.off_status + sizeof(int32_t) - w.off_counters;
     w.off_part_lse = (w.off_status + sizeof(int32_t) + 255) / 256 * 256;

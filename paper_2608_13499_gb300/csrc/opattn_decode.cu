@@ -13,26 +13,32 @@
 // token c / G, head c % G of the kv head.  The kernel is bound by HBM: each
 // K/V byte is read once and feeds 2 * G * Lq flops.
 //
-// Softmax runs per column over the keys of a tile, one key per thread of the
-// softmax warpgroup (one TMEM lane each).  The subtraction base of a column
+// Softmax runs per column over the keys of a tile, one key per thread (one
+// TMEM lane each).  Two softmax warpgroups split the columns: warpgroup w
+// owns columns [w * H, w * H + H) of every tile, and both warpgroups' warps
+// i and 4 + i read TMEM lane quarter i.  The subtraction base of a column
 // is the exact maximum of the chunk's first tile and is reused while no
 // score exceeds it by more than 2^kRebaseSlack; a larger score makes the
 // warpgroup take the tile's exact maximum and rescale the running sums and
 // the O accumulator.  Long key ranges are split into chunks (split-KV); a
 // chunk writes its normalised partial O and its log2-domain LSE, and the
 // last chunk of a (sequence, kv head) to finish merges the partials with
-// LSE weights.
+// LSE weights; each warpgroup counts and merges its own columns.
 //
-// CTA layout (192 threads, one CTA per SM, persistent over its unit list):
-//   warps 0-3  softmax / epilogue / merge (thread t = TMEM lane t)
-//   warp 4     TMA producer: Q^T of the unit, then K_j and V_j
-//   warp 5     TMEM owner + MMA issuer (whole warp, one elected lane issues)
-// TMEM (128 columns): S0 | S1 (32 fp32 columns each) | O (32 columns).
+// CTA layout (352 threads, one CTA per SM, persistent over its unit list):
+//   warps 0-3  softmax / epilogue / merge of columns [0, H)
+//   warps 4-7  the same for columns [H, 2H) (thread t of a warpgroup = TMEM lane t)
+//   warp 8     TMA producer: Q^T of the unit, then its K tiles
+//   warp 9     TMEM owner + MMA issuer (whole warp, one elected lane issues)
+//   warp 10    TMA producer of the V tiles
+// TMEM (128 columns): S0 | S1 | S2 (32 fp32 columns each) | O (32 columns).
 //
-// MMA order (tiles counted across the CTA's units as g):
-//   S(0), S(1), then per tile: wait P(g), PV(g), S(g + 2)
-// S(g + 2) reuses the S buffer of tile g only after PV(g), i.e. after the
-// softmax warps have read S(g) and written P(g).
+// MMA order within a unit of n tiles (tiles counted across the CTA's units
+// as g; S buffer g mod 3, P buffer g mod 2):
+//   S(0), S(1), S(2), then per tile: wait P(g), PV(g), S(g + 3)
+// S(g + 3) reuses the S buffer of tile g only after P(g) has arrived, i.e.
+// after the softmax warps have read S(g); the three S buffers keep the MMA
+// round trip off the softmax warps' critical path.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -50,10 +56,11 @@ namespace {
 constexpr int D = kDecHeadDim;
 constexpr int NC = kDecCols;
 constexpr int kTile = 128;  // keys per K/V tile
-constexpr int kThreadsDec = 192;
-constexpr int kWarpProducerDec = 4;
-constexpr int kWarpMmaDec = 5;
-constexpr uint32_t kBarWG = 1;        // named barrier of the softmax warpgroup
+constexpr int kThreadsDec = 352;
+constexpr int kWarpProducerDec = 8;   // Q^T and K
+constexpr int kWarpMmaDec = 9;
+constexpr int kWarpProducerVDec = 10;  // V
+constexpr uint32_t kBarWG0 = 1;       // named barrier of softmax warpgroup w: kBarWG0 + w
 constexpr uint32_t kWGThreads = 128;
 // A score may exceed its column's subtraction base by up to 2^24 in the
 // exponential before the base is moved: fp32 sums of up to 2^31 keys and the
@@ -72,8 +79,8 @@ struct DCfg {
     static constexpr int kKOff = 2 * kQBytes;
     static constexpr int kVOff = kKOff + kKSlots * kSlotBytes;
     static constexpr int kPOff = kVOff + kVSlots * kSlotBytes;  // two P buffers (tile parity)
-    static constexpr int kRedOff = kPOff + 2 * kPBytes;         // two [4 warps][32] float buffers
-    static constexpr int kRedBytes = 2 * 4 * 32 * 4;
+    static constexpr int kRedOff = kPOff + 2 * kPBytes;         // per warpgroup two [4 warps][16] floats
+    static constexpr int kRedBytes = 2 * 2 * 4 * 16 * 4;
     static constexpr int kBarOff = kRedOff + kRedBytes;
     static constexpr int kBarKFull = 0;
     static constexpr int kBarKEmpty = kKSlots;
@@ -81,8 +88,9 @@ struct DCfg {
     static constexpr int kBarVEmpty = 2 * kKSlots + kVSlots;
     static constexpr int kBarQFull = 2 * kKSlots + 2 * kVSlots;  // + Q buffer
     static constexpr int kBarQEmpty = kBarQFull + 2;
+    static constexpr int kSBufs = 3;
     static constexpr int kBarSFull = kBarQEmpty + 2;   // + S buffer
-    static constexpr int kBarPFull = kBarSFull + 2;    // + P buffer
+    static constexpr int kBarPFull = kBarSFull + kSBufs;  // + P buffer
     static constexpr int kBarPVDone = kBarPFull + 2;   // + P buffer: PV of that buffer's tile complete
     static constexpr int kBarDrain = kBarPVDone + 2;
     static constexpr int kBarNever = kBarDrain + 1;
@@ -91,7 +99,7 @@ struct DCfg {
     static constexpr int kSmemBytes = kMiscOff + 16 + 1024;  // + slack for 1024-byte alignment
     static constexpr uint32_t kTmemCols = 128;
     static constexpr uint32_t kColS = 0;  // + 32 * S buffer
-    static constexpr uint32_t kColO = 64;
+    static constexpr uint32_t kColO = 96;
     // S^T = K . Q^T: A = K tile (K-major), B = Q^T rows (K-major).
     static constexpr uint32_t kIdescS = ptx::idesc_bf16_f32_ab(kTile, NC, false, false);
     // O^T = V^T . P^T: A = V tile read channel-major (MN-major), B = P^T rows (K-major).
@@ -115,72 +123,67 @@ struct DParams {
     uint32_t flags;
 };
 
-__device__ __forceinline__ void dec_producer(const CUtensorMap* tmQ, const CUtensorMap* tmK, const CUtensorMap* tmV,
-                                             const DParams& p, int ubeg, int uend, uint32_t sQ, uint32_t sK,
-                                             uint32_t sV, uint32_t sBar, volatile int32_t* abort_flag) {
+// TMA producers.  One thread loads the unit's Q^T and its K tiles, another
+// its V tiles, so that K loads run ahead as far as the K ring allows and are
+// never held behind a V slot (V(j) is freed only by PV(j), K(j) already by
+// S(j)).
+template <bool kIsV>
+__device__ __forceinline__ void dec_producer(const CUtensorMap* tmQ, const CUtensorMap* tmKV, const DParams& p,
+                                             int ubeg, int uend, uint32_t sQ, uint32_t sRing, uint32_t sBar,
+                                             volatile int32_t* abort_flag) {
     using C = DCfg;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    constexpr int kSlots = kIsV ? C::kVSlots : C::kKSlots;
+    constexpr int kFull = kIsV ? C::kBarVFull : C::kBarKFull;
+    constexpr int kEmpty = kIsV ? C::kBarVEmpty : C::kBarKEmpty;
     const uint64_t once = ptx::policy_evict_first();  // every K/V byte is read once
-    uint32_t kslot = 0, kpar = 0, vslot = 0, vpar = 0;
-    uint32_t k_issued = 0, v_issued = 0, items = 0;
+    uint32_t slot = 0, par = 0, issued = 0, items = 0;
     uint32_t q_issued[2] = {0u, 0u};
     bool aborted = false;
     for (int ui = ubeg; ui < uend && !aborted; ++ui) {
         const DecUnit u = p.units[ui];
         if (u.n_tiles <= 0) continue;
-        const int qb = static_cast<int>(items & 1u);
-        if (!bounded_wait(bar(C::kBarQEmpty + qb), (q_issued[qb] & 1u) ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
-            aborted = true;
-            break;
+        if (!kIsV) {
+            const int qb = static_cast<int>(items & 1u);
+            if (!bounded_wait(bar(C::kBarQEmpty + qb), (q_issued[qb] & 1u) ^ 1u, abort_flag, p.status,
+                              kWaitLimitNs)) {
+                aborted = true;
+                break;
+            }
+            ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + qb), C::kQBytes);
+#pragma unroll
+            for (int b = 0; b < 2; ++b)
+                ptx::tma_load_3d(sQ + qb * C::kQBytes + b * (NC * 128), tmQ, bar(C::kBarQFull + qb), b * 64,
+                                 u.kvh * p.G, u.q_tok0);
+            ++q_issued[qb];
+            ++items;
         }
-        ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + qb), C::kQBytes);
-#pragma unroll
-        for (int b = 0; b < 2; ++b)
-            ptx::tma_load_3d(sQ + qb * C::kQBytes + b * (NC * 128), tmQ, bar(C::kBarQFull + qb), b * 64,
-                             u.kvh * p.G, u.q_tok0);
-        ++q_issued[qb];
-        ++items;
-        for (int j = 0; j < u.n_tiles && !aborted; ++j) {
+        for (int j = 0; j < u.n_tiles; ++j) {
             const int row = u.k_row0 + (u.tile0 + j) * kTile;
-            if (!bounded_wait(bar(C::kBarKEmpty + kslot), kpar ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
+            if (!bounded_wait(bar(kEmpty + slot), par ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
                 aborted = true;
                 break;
             }
-            ptx::mbar_arrive_expect_tx(bar(C::kBarKFull + kslot), C::kSlotBytes);
+            ptx::mbar_arrive_expect_tx(bar(kFull + slot), C::kSlotBytes);
 #pragma unroll
             for (int b = 0; b < 2; ++b)
-                ptx::tma_load_3d_hint(sK + kslot * C::kSlotBytes + b * (kTile * 128), tmK, bar(C::kBarKFull + kslot),
+                ptx::tma_load_3d_hint(sRing + slot * C::kSlotBytes + b * (kTile * 128), tmKV, bar(kFull + slot),
                                       b * 64, u.kvh, row, once);
-            ++k_issued;
-            if (++kslot == C::kKSlots) { kslot = 0; kpar ^= 1u; }
-            if (!bounded_wait(bar(C::kBarVEmpty + vslot), vpar ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
-                aborted = true;
-                break;
-            }
-            ptx::mbar_arrive_expect_tx(bar(C::kBarVFull + vslot), C::kSlotBytes);
-#pragma unroll
-            for (int b = 0; b < 2; ++b)
-                ptx::tma_load_3d_hint(sV + vslot * C::kSlotBytes + b * (kTile * 128), tmV, bar(C::kBarVFull + vslot),
-                                      b * 64, u.kvh, row, once);
-            ++v_issued;
-            if (++vslot == C::kVSlots) { vslot = 0; vpar ^= 1u; }
+            ++issued;
+            if (++slot == kSlots) { slot = 0; par ^= 1u; }
         }
     }
     if (aborted) {
         // Let every copy still in flight land before the CTA exits: at most
         // one outstanding load per slot and per Q buffer (the latest).
-        for (uint32_t s = 0; s < static_cast<uint32_t>(C::kKSlots); ++s)
-            if (k_issued > s) {
-                const uint32_t uses = (k_issued - s + C::kKSlots - 1) / C::kKSlots;
-                drain_wait(bar(C::kBarKFull + s), (uses - 1u) & 1u, kDrainLimitNs);
+        for (uint32_t s = 0; s < static_cast<uint32_t>(kSlots); ++s)
+            if (issued > s) {
+                const uint32_t uses = (issued - s + kSlots - 1) / kSlots;
+                drain_wait(bar(kFull + s), (uses - 1u) & 1u, kDrainLimitNs);
             }
-        for (uint32_t s = 0; s < static_cast<uint32_t>(C::kVSlots); ++s)
-            if (v_issued > s) {
-                const uint32_t uses = (v_issued - s + C::kVSlots - 1) / C::kVSlots;
-                drain_wait(bar(C::kBarVFull + s), (uses - 1u) & 1u, kDrainLimitNs);
-            }
-        for (int i = 0; i < 2; ++i)
-            if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
+        if (!kIsV)
+            for (int i = 0; i < 2; ++i)
+                if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
     }
 }
 
@@ -193,6 +196,7 @@ __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, ui
         return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
     };
     uint32_t kslot = 0, kpar = 0, vslot = 0, vpar = 0, items = 0, g = 0;
+    uint32_t sbuf = 0;  // S buffer of the next S MMA (tiles are scored in order)
     uint32_t q_uses[2] = {0u, 0u};
     bool ok = true;
     if (p.flags & kFlagForceTimeout)
@@ -207,8 +211,8 @@ __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, ui
         ++q_uses[qb];
         ++items;
         const uint32_t qaddr = sQ + qb * C::kQBytes;
-        // S(gg) = K . Q^T from the next K slot into S buffer gg & 1.
-        auto issue_s = [&](uint32_t gg) -> bool {
+        // S = K . Q^T from the next K slot into the next S buffer.
+        auto issue_s = [&]() -> bool {
             if (!wait(C::kBarKFull + kslot, kpar)) return false;
             ptx::tc_fence_after();
             const uint32_t kaddr = sK + kslot * C::kSlotBytes;
@@ -216,17 +220,19 @@ __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, ui
             for (int ks = 0; ks < D / 16; ++ks) {
                 const uint32_t aoff = (ks >> 2) * (kTile * 128) + (ks & 3) * 32;
                 const uint32_t boff = (ks >> 2) * (NC * 128) + (ks & 3) * 32;
-                ptx::mma_ss_warp(tmem + C::kColS + 32u * (gg & 1u), ptx::sdesc_sw128(kaddr + aoff, 16, 1024),
+                ptx::mma_ss_warp(tmem + C::kColS + 32u * sbuf, ptx::sdesc_sw128(kaddr + aoff, 16, 1024),
                                  ptx::sdesc_sw128(qaddr + boff, 16, 1024), C::kIdescS, ks > 0 ? 1u : 0u);
             }
-            ptx::tc_commit_warp(bar(C::kBarSFull + static_cast<int>(gg & 1u)));
+            ptx::tc_commit_warp(bar(C::kBarSFull + static_cast<int>(sbuf)));
             ptx::tc_commit_warp(bar(C::kBarKEmpty + kslot));
             if (++kslot == C::kKSlots) { kslot = 0; kpar ^= 1u; }
+            if (++sbuf == C::kSBufs) sbuf = 0;
             return true;
         };
-        if (!(ok = issue_s(g))) break;
-        if (n > 1 && !(ok = issue_s(g + 1))) break;
-        if (n <= 2) ptx::tc_commit_warp(bar(C::kBarQEmpty + qb));
+        const int pre = n < C::kSBufs ? n : C::kSBufs;
+        for (int i = 0; i < pre && ok; ++i) ok = issue_s();
+        if (!ok) break;
+        if (n <= C::kSBufs) ptx::tc_commit_warp(bar(C::kBarQEmpty + qb));
         for (int j = 0; j < n; ++j) {
             const uint32_t gj = g + static_cast<uint32_t>(j);
             const int pb = static_cast<int>(gj & 1u);
@@ -247,9 +253,9 @@ __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, ui
             ptx::tc_commit_warp(bar(C::kBarPVDone + pb));
             ptx::tc_commit_warp(bar(C::kBarVEmpty + vslot));
             if (++vslot == C::kVSlots) { vslot = 0; vpar ^= 1u; }
-            if (j + 2 < n) {
-                if (!(ok = issue_s(gj + 2))) break;
-                if (j + 3 == n) ptx::tc_commit_warp(bar(C::kBarQEmpty + qb));
+            if (j + C::kSBufs < n) {
+                if (!(ok = issue_s())) break;
+                if (j + C::kSBufs + 1 == n) ptx::tc_commit_warp(bar(C::kBarQEmpty + qb));
             }
         }
         g += static_cast<uint32_t>(n);
@@ -259,14 +265,15 @@ __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, ui
     drain_wait(bar(C::kBarDrain), 0u, kDrainLimitNs);
 }
 
-// Reduces v[c] over the 128 threads of the softmax warpgroup for each of the
+// Reduces v[c] over the 128 threads of a softmax warpgroup for each of its
 // NCOL columns and gives every thread all NCOL results.  Within a warp, lanes
 // 8, 16, ... apart are first combined column by column until NCOL lanes are
 // left per column; the columns are then halved with butterfly exchanges, so
 // lane l ends with column l mod NCOL.  The four warps combine through shared
 // memory.
 template <int NCOL, bool kMax>
-__device__ __forceinline__ void wg_reduce(const float* v, float* out, float* red, int warp, int lane) {
+__device__ __forceinline__ void wg_reduce(const float* v, float* out, float* red, int warp, int lane,
+                                          uint32_t bar_id) {
     float x[NCOL];
 #pragma unroll
     for (int c = 0; c < NCOL; ++c) x[c] = v[c];
@@ -289,11 +296,13 @@ __device__ __forceinline__ void wg_reduce(const float* v, float* out, float* red
             x[i] = kMax ? fmaxf(keep, recv) : keep + recv;
         }
     }
-    red[warp * 32 + lane] = x[0];
-    ptx::bar_sync(kBarWG, kWGThreads);
-    float t = red[lane];
+    static_assert(NCOL <= 16, "one warpgroup reduces at most 16 columns");
+    if (lane < NCOL) red[warp * 16 + lane] = x[0];
+    ptx::bar_sync(bar_id, kWGThreads);
+    const int col = lane & (NCOL - 1);
+    float t = red[col];
 #pragma unroll
-    for (int w = 1; w < 4; ++w) t = kMax ? fmaxf(t, red[w * 32 + lane]) : t + red[w * 32 + lane];
+    for (int w = 1; w < 4; ++w) t = kMax ? fmaxf(t, red[w * 16 + col]) : t + red[w * 16 + col];
 #pragma unroll
     for (int c = 0; c < NCOL; ++c) out[c] = __shfl_sync(0xFFFFFFFFu, t, c);
 }
@@ -306,27 +315,35 @@ __device__ __forceinline__ int64_t out_row(const DParams& p, const DecUnit& u, i
     return static_cast<int64_t>(u.q_tok0 + (c >> p.g_shift)) * p.Hq + u.kvh * p.G + (c & (p.G - 1));
 }
 
-// Softmax warpgroup.  NCOL (8, 16 or 32) is the number of S^T / O^T columns
-// it processes: the largest G * Lq of the batch rounded up.  Columns beyond
-// a unit's own G * Lq are masked and never written to P^T (zero there).
+// Softmax warpgroup `wg` (0 or 1).  NCOL (4, 8 or 16) is the number of
+// S^T / O^T columns each warpgroup processes: half the largest G * Lq of the
+// batch, rounded up.  Columns beyond a unit's own G * Lq are masked and never
+// written to P^T (zero there).  `tid` is the thread's index in its
+// warpgroup, which is also its TMEM lane and the key of the tile it scores.
 template <int NCOL>
 __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sP,
-                                            float* sRed, uint32_t sBar, int tid, volatile int32_t* abort_flag) {
+                                            float* sRed, uint32_t sBar, int wg, int tid,
+                                            volatile int32_t* abort_flag) {
     using C = DCfg;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
     const int warp = tid >> 5, lane = tid & 31;
+    const uint32_t kBarWG = kBarWG0 + static_cast<uint32_t>(wg);
+    const int col0 = wg * NCOL;  // first column of this warpgroup
     const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
-    const uint32_t tS = tmem + lane_off + C::kColS;
-    const uint32_t tO = tmem + lane_off + C::kColO;
+    const uint32_t tS = tmem + lane_off + C::kColS + static_cast<uint32_t>(col0);
+    const uint32_t tO = tmem + lane_off + C::kColO + static_cast<uint32_t>(col0);
+    sRed += wg * 128;
     const float cl = p.scale_log2;
     const int gs = p.g_shift;
     // P^T element (column c, key tid): 64-key block, row c, 16-byte chunk swizzled by c mod 8.
-    const uint32_t p_thread = static_cast<uint32_t>((tid >> 6) * (NC * 128) + ((tid & 7) << 1));
+    // A lane pair (keys 2i, 2i + 1) writes one 32-bit word per column.
+    const uint32_t p_pair = static_cast<uint32_t>((tid >> 6) * (NC * 128) + col0 * 128 + ((tid & 6) << 1));
     const uint32_t p_chunk = static_cast<uint32_t>((tid & 63) >> 3);
     uint32_t g = 0;
+    uint32_t sbuf = 0, spar = 0;  // S buffer of tile g (g mod 3) and its phase parity
     int red_buf = 0;
     auto red_ptr = [&]() {
-        float* r = sRed + red_buf * 128;
+        float* r = sRed + red_buf * 64;
         red_buf ^= 1;
         return r;
     };
@@ -343,8 +360,8 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
         if (u.n_tiles <= 0) {  // the sequence has no key: O = 0, LSE = -inf
 #pragma unroll
             for (int c = 0; c < NCOL; ++c) {
-                if (c >= ncols) break;
-                const int64_t row = out_row(p, u, c);
+                if (col0 + c >= ncols) break;
+                const int64_t row = out_row(p, u, col0 + c);
                 p.o[row * D + tid] = 0;
                 if (tid == c) p.lse[row] = -INFINITY;
             }
@@ -361,20 +378,20 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
         for (int j = 0; j < u.n_tiles; ++j) {
             const uint32_t b = g & 1u;
             // S(g) ready, and P buffer b free (last read by PV(g - 2)).
-            bool ok = warp_wait(C::kBarSFull + static_cast<int>(b), (g >> 1) & 1u);
+            bool ok = warp_wait(C::kBarSFull + static_cast<int>(sbuf), spar);
             if (ok && g >= 2u) ok = warp_wait(C::kBarPVDone + static_cast<int>(b), ((g - 2u) >> 1) & 1u);
             float s[NCOL];
             bool need = j == 0;
             if (ok) {
                 ptx::tc_fence_after();
                 uint32_t sr[NCOL];
-                ptx::tmem_ld_n<NCOL>(tS + 32u * b, sr);
+                ptx::tmem_ld_n<NCOL>(tS + 32u * sbuf, sr);
                 ptx::tmem_wait_ld();
                 ptx::tmem_ld_fence<NCOL>(sr);
                 const int key = (u.tile0 + j) * kTile + tid;
 #pragma unroll
                 for (int c = 0; c < NCOL; ++c) {
-                    const bool vis = c < ncols && key <= lim0 + (c >> gs);
+                    const bool vis = col0 + c < ncols && key <= lim0 + ((col0 + c) >> gs);
                     s[c] = vis ? __uint_as_float(sr[c]) * cl : -INFINITY;
                     need |= s[c] - base[c] > kRebaseSlack;
                 }
@@ -384,7 +401,7 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
             if (ptx::bar_red_or(kBarWG, kWGThreads, need || !ok)) {
                 if (!ptx::bar_red_and(kBarWG, kWGThreads, ok)) return;
                 float tmax[NCOL];
-                wg_reduce<NCOL, true>(s, tmax, red_ptr(), warp, lane);
+                wg_reduce<NCOL, true>(s, tmax, red_ptr(), warp, lane, kBarWG);
                 bool scaled = false;
                 float alpha[NCOL];
 #pragma unroll
@@ -413,19 +430,37 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
                     ptx::tmem_wait_st();
                 }
             }
-            const uint32_t pbase = sP + b * C::kPBytes + p_thread;
+            uint32_t pk[NCOL];
 #pragma unroll
             for (int c = 0; c < NCOL; ++c) {
                 const float pv = ptx::ex2_approx(s[c] - (base[c] == -INFINITY ? 0.f : base[c]));
-                const uint32_t pk = ptx::pack_bf16x2(pv, 0.f);
+                pk[c] = ptx::pack_bf16x2(pv, 0.f) & 0xFFFFu;
                 l[c] += pv;
-                lh[c] += ptx::bf16lo_to_f32(pk);
-                if (c < ncols) ptx::st_shared_u16(pbase + c * 128 + ((p_chunk ^ (c & 7)) << 4), static_cast<uint16_t>(pk));
+                lh[c] += ptx::bf16lo_to_f32(pk[c]);
+            }
+            // P^T stores as 32-bit words of two adjacent keys: the even lane of
+            // a pair writes column c, the odd lane column c ^ kPair, each after
+            // one exchange.  With kPair = 4 the two rows a warp writes land in
+            // opposite halves of the banks (the swizzle moves row c's chunks
+            // by c mod 8), so a warp stores 128 bytes with no conflict.
+            // Masked columns hold p = 0, so all NCOL columns are written.
+            constexpr int kPair = NCOL >= 8 ? 4 : 1;
+            const bool odd = (lane & 1) != 0;
+            const uint32_t prow = sP + b * C::kPBytes + p_pair;
+#pragma unroll
+            for (int c = 0; c < NCOL; ++c) {
+                if (c & kPair) continue;
+                const int c2 = c | kPair;
+                const uint32_t recv = __shfl_xor_sync(0xFFFFFFFFu, odd ? pk[c] : pk[c2], 1);
+                const int cw = odd ? c2 : c;  // column this lane writes
+                const uint32_t word = odd ? (recv | (pk[c2] << 16)) : (pk[c] | (recv << 16));
+                ptx::st_shared_u32(prow + cw * 128 + ((p_chunk ^ ((col0 + cw) & 7)) << 4), word);
             }
             ptx::fence_proxy_async_smem();
             ptx::tc_fence_before();
             ptx::mbar_arrive(bar(C::kBarPFull + static_cast<int>(b)));
             ++g;
+            if (++sbuf == C::kSBufs) { sbuf = 0; spar ^= 1u; }
         }
         // epilogue: wait for the unit's last PV
         const uint32_t gl = g - 1u;
@@ -436,15 +471,15 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
         ptx::tmem_wait_ld();
         ptx::tmem_ld_fence<NCOL>(ov);
         float L[NCOL], LH[NCOL];
-        wg_reduce<NCOL, false>(l, L, red_ptr(), warp, lane);
-        wg_reduce<NCOL, false>(lh, LH, red_ptr(), warp, lane);
+        wg_reduce<NCOL, false>(l, L, red_ptr(), warp, lane, kBarWG);
+        wg_reduce<NCOL, false>(lh, LH, red_ptr(), warp, lane, kBarWG);
         if (u.part < 0) {
             // O is normalised by the sum of the rounded weights the PV MMA
             // used (a weighted mean of V rows); LSE uses the unrounded sum.
 #pragma unroll
             for (int c = 0; c < NCOL; ++c) {
-                if (c >= ncols) break;
-                const int64_t row = out_row(p, u, c);
+                if (col0 + c >= ncols) break;
+                const int64_t row = out_row(p, u, col0 + c);
                 const float inv = LH[c] > 0.f ? 1.f / LH[c] : 0.f;
                 p.o[row * D + tid] = f32_to_bf16_bits(__uint_as_float(ov[c]) * inv);
                 if (tid == c) p.lse[row] = L[c] > 0.f ? (base[c] + log2f(L[c])) * kLn2Dec : -INFINITY;
@@ -455,21 +490,22 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
         float* po = p.part_o + static_cast<int64_t>(u.part) * NC * D;
 #pragma unroll
         for (int c = 0; c < NCOL; ++c) {
-            if (c >= ncols) break;
-            po[c * D + tid] = LH[c] > 0.f ? __uint_as_float(ov[c]) / LH[c] : 0.f;
-            if (tid == c) p.part_lse[u.part * NC + c] = L[c] > 0.f ? base[c] + log2f(L[c]) : -INFINITY;
+            if (col0 + c >= ncols) break;
+            po[(col0 + c) * D + tid] = LH[c] > 0.f ? __uint_as_float(ov[c]) / LH[c] : 0.f;
+            if (tid == c) p.part_lse[u.part * NC + col0 + c] = L[c] > 0.f ? base[c] + log2f(L[c]) : -INFINITY;
         }
         __threadfence();
         ptx::bar_sync(kBarWG, kWGThreads);
         bool last = false;
-        if (tid == 0) last = atomicAdd(p.counters + u.group, 1) == u.n_chunks - 1;
+        // Each warpgroup counts the chunks of its own columns.
+        if (tid == 0) last = atomicAdd(p.counters + 2 * u.group + wg, 1) == u.n_chunks - 1;
         last = ptx::bar_red_or(kBarWG, kWGThreads, last);
         if (!last) continue;
         // This unit finished last: merge the (sequence, kv head)'s partials,
         // O = sum_k 2^(lse_k - lse) O_k with lse = log2 sum_k 2^lse_k.
         __threadfence();
         const int part0 = u.part - u.chunk;
-        for (int c = 0; c < ncols; ++c) {
+        for (int c = col0; c < min(col0 + NCOL, ncols); ++c) {
             float m = -INFINITY;
             for (int k = 0; k < u.n_chunks; ++k) m = fmaxf(m, __ldcg(p.part_lse + (part0 + k) * NC + c));
             float acc = 0.f, wsum = 0.f;
@@ -518,11 +554,11 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
             ptx::mbar_init(sBar + 8u * (C::kBarVFull + i), 1);
             ptx::mbar_init(sBar + 8u * (C::kBarVEmpty + i), 1);
         }
+        for (int i = 0; i < C::kSBufs; ++i) ptx::mbar_init(sBar + 8u * (C::kBarSFull + i), 1);
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(sBar + 8u * (C::kBarQFull + i), 1);
             ptx::mbar_init(sBar + 8u * (C::kBarQEmpty + i), 1);
-            ptx::mbar_init(sBar + 8u * (C::kBarSFull + i), 1);
-            ptx::mbar_init(sBar + 8u * (C::kBarPFull + i), kWGThreads);
+            ptx::mbar_init(sBar + 8u * (C::kBarPFull + i), 2 * kWGThreads);
             ptx::mbar_init(sBar + 8u * (C::kBarPVDone + i), 1);
         }
         ptx::mbar_init(sBar + 8u * C::kBarDrain, 1);
@@ -530,11 +566,12 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
         *abort_flag = 0;
         ptx::fence_mbar_init();
     }
-    if (tid < static_cast<int>(kWGThreads)) {
+    if (tid < static_cast<int>(2 * kWGThreads)) {
         // Columns a unit does not use are never written: start them finite.
-        const uint32_t dst = sP + static_cast<uint32_t>(tid) * (2 * C::kPBytes / kWGThreads);
+        constexpr int kPer = 2 * C::kPBytes / (2 * static_cast<int>(kWGThreads));
+        const uint32_t dst = sP + static_cast<uint32_t>(tid) * kPer;
 #pragma unroll
-        for (int i = 0; i < 2 * C::kPBytes / static_cast<int>(kWGThreads); i += 16) ptx::st_shared_v4(dst + i, 0u, 0u, 0u, 0u);
+        for (int i = 0; i < kPer; i += 16) ptx::st_shared_v4(dst + i, 0u, 0u, 0u, 0u);
         ptx::fence_proxy_async_smem();
     }
     if (warp == kWarpMmaDec) {
@@ -544,8 +581,8 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
     if (warp == kWarpProducerDec && lane == 0) {
         ptx::prefetch_tmap(&tmQ);
         ptx::prefetch_tmap(&tmK);
-        ptx::prefetch_tmap(&tmV);
     }
+    if (warp == kWarpProducerVDec && lane == 0) ptx::prefetch_tmap(&tmV);
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
@@ -553,10 +590,13 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
     const int ubeg = p.cta_off[blockIdx.x];
     const int uend = p.cta_off[blockIdx.x + 1];
 
-    if (warp < 4) {
-        dec_softmax<NCOL>(p, ubeg, uend, tmem, sP, sRed, sBar, tid, abort_flag);
+    if (warp < 8) {
+        dec_softmax<NCOL>(p, ubeg, uend, tmem, sP, sRed, sBar, warp >> 2, tid & 127, abort_flag);
     } else if (warp == kWarpProducerDec) {
-        if (lane == 0) dec_producer(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sK, sV, sBar, abort_flag);
+        if (lane == 0) dec_producer<false>(&tmQ, &tmK, p, ubeg, uend, sQ, sK, sBar, abort_flag);
+        __syncwarp();
+    } else if (warp == kWarpProducerVDec) {
+        if (lane == 0) dec_producer<true>(&tmQ, &tmV, p, ubeg, uend, sQ, sV, sBar, abort_flag);
         __syncwarp();
     } else if (warp == kWarpMmaDec) {
         dec_mma(p, ubeg, uend, tmem, sQ, sK, sV, sP, sBar, abort_flag);
@@ -622,9 +662,10 @@ int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream) {
     kp.part_lse = a.part_lse;
     kp.status = a.status;
     kp.flags = a.flags;
-    if (a.max_cols <= 8) return launch_ncol<8>(a, tq, tk, tv, kp, stream);
-    if (a.max_cols <= 16) return launch_ncol<16>(a, tq, tk, tv, kp, stream);
-    return launch_ncol<32>(a, tq, tk, tv, kp, stream);
+    // columns per softmax warpgroup
+    if (a.max_cols <= 8) return launch_ncol<4>(a, tq, tk, tv, kp, stream);
+    if (a.max_cols <= 16) return launch_ncol<8>(a, tq, tk, tv, kp, stream);
+    return launch_ncol<16>(a, tq, tk, tv, kp, stream);
 }
 
 }  // namespace opattn

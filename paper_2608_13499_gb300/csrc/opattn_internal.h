@@ -106,7 +106,7 @@ struct DecodeLaunchArgs {
     const int32_t* cta_off;   // device, n_cta + 1
     int32_t n_cta;
     int32_t max_cols;         // largest G * Lq of the batch (<= kDecCols)
-    int32_t* counters;        // device, one per split (sequence, kv head), zero at launch
+    int32_t* counters;        // device, two per split (sequence, kv head), zero at launch
     float* part_o;            // device, [parts][kDecCols][kDecHeadDim]
     float* part_lse;          // device, [parts][kDecCols] (log2 domain)
     int32_t* status;          // device

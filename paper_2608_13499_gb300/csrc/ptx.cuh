@@ -199,18 +199,32 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r) {
                  "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
                  : "memory");
 }
-// N (8, 16 or 32) consecutive columns.
+__device__ __forceinline__ void tmem_ld4(uint32_t taddr, uint32_t* r) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t* r) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3])
+                 : "memory");
+}
+// N (4, 8, 16 or 32) consecutive columns.
 template <int N>
 __device__ __forceinline__ void tmem_ld_n(uint32_t taddr, uint32_t* r) {
+    static_assert(N == 4 || N == 8 || N == 16 || N == 32, "tmem_ld_n");
     if constexpr (N == 32) tmem_ld32(taddr, r);
     else if constexpr (N == 16) tmem_ld16(taddr, r);
-    else tmem_ld8(taddr, r);
+    else if constexpr (N == 8) tmem_ld8(taddr, r);
+    else tmem_ld4(taddr, r);
 }
 template <int N>
 __device__ __forceinline__ void tmem_st_n(uint32_t taddr, const uint32_t* r) {
+    static_assert(N == 4 || N == 8 || N == 16 || N == 32, "tmem_st_n");
     if constexpr (N == 32) tmem_st32(taddr, r);
     else if constexpr (N == 16) tmem_st16(taddr, r);
-    else tmem_st8(taddr, r);
+    else if constexpr (N == 8) tmem_st8(taddr, r);
+    else tmem_st4(taddr, r);
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
@@ -282,6 +296,9 @@ __device__ __forceinline__ bool bar_red_and(uint32_t id, uint32_t count, bool x)
 }
 __device__ __forceinline__ void st_shared_u16(uint32_t addr, uint16_t v) {
     asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
+}
+__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
