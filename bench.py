@@ -272,10 +272,33 @@ def run_ours(args, w):
     stream = torch.cuda.current_stream(dev)
 
     decode = is_decode(w)
-    plan = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=decode)
-    one_shot = pkg.opattn_decode if decode else pkg.opattn_prefill
+    paged = w.page_size > 0
+    if paged:
+        # K/V live in a paged cache (shuffled pages); the packed copies are only the source.
+        lay = W.paged_layout(w.k_lens, w.page_size, seed=w.seed)
+        k_packed, v_packed = k, v
+        k, v = W.to_paged(k, w.k_lens, lay), W.to_paged(v, w.k_lens, lay)
+        table = torch.from_numpy(lay.block_table).to(dev)
+        seqlens_k = np.asarray(w.k_lens, dtype=np.int32)
+        plan = pkg.Plan(w.cu_q, seqlens_k, w.Hq, w.Hkv, w.d, block_size=w.page_size, max_blocks=lay.max_blocks)
+
+        def run_plan():
+            plan.run_paged(q, k, v, table, lay.num_blocks, o, lse, w.scale, stream)
+
+        def one_shot(dq, dk, dv):
+            pkg.opattn_decode_paged(dq, dk, dv, table, lay.num_blocks, lay.page_size, lay.max_blocks, o, lse,
+                                    w.cu_q, seqlens_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
+    else:
+        plan = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=decode)
+        call = pkg.opattn_decode if decode else pkg.opattn_prefill
+
+        def run_plan():
+            plan.run(q, k, v, o, lse, w.scale, stream)
+
+        def one_shot(dq, dk, dv):
+            call(dq, dk, dv, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
     for _ in range(max(args.warmup, 3)):
-        plan.run(q, k, v, o, lse, w.scale, stream)
+        run_plan()
     torch.cuda.synchronize(dev)
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
@@ -289,7 +312,7 @@ def run_ours(args, w):
     t_start.record(stream)
     for i in range(args.steps):
         ev[i][0].record(stream)
-        plan.run(q, k, v, o, lse, w.scale, stream)
+        run_plan()
         ev[i][1].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize(dev)
@@ -316,7 +339,7 @@ def run_ours(args, w):
         dq.copy_(hq, non_blocking=True)
         dk.copy_(hk, non_blocking=True)
         dv.copy_(hv, non_blocking=True)
-        one_shot(dq, dk, dv, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream)
+        one_shot(dq, dk, dv)
         ho.copy_(o, non_blocking=True)
         hl.copy_(lse, non_blocking=True)
 
@@ -334,13 +357,13 @@ def run_ours(args, w):
     e2e_elapsed, e2e_flops = aggregate_over_ranks(e0.elapsed_time(e1) / 1e3, float(flops) * e2e_steps,
                                                   dist if world > 1 else None)
     e2e_value = e2e_flops / e2e_elapsed / 1e12
-    h2d = q.numel() * 2 + k.numel() * 2 + v.numel() * 2
+    h2d = q.numel() * 2 + k.numel() * 2 + v.numel() * 2  # for a paged cache: the whole cache
     d2h = o.numel() * 2 + lse.numel() * 4
     plan.close()
 
     cpu_base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        qc, kc, vc = hq, hk, hv
+        qc, kc, vc = (hq, hk, hv) if not paged else (hq, k_packed.cpu(), v_packed.cpu())
         r = oracle_sample(w, qc, kc, vc, args.cpu_seconds)
         cpu_base = {"value": r["flops"] / r["seconds"] / 1e12, "unit": "TFLOP/s", "cores": r["threads"],
                     "kind": "oracle",
@@ -427,7 +450,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama3_70b",
                     help="tiny | llama3_8b | llama3_70b | bursty | chunked | decode_llama3_70b | "
-                         "decode_llama3_8b | decode_spec4_llama3_70b")
+                         "decode_llama3_8b | decode_spec4_llama3_70b | decode_llama3_70b_paged16")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")

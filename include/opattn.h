@@ -213,6 +213,38 @@ OPATTN_API opattn_status opattn_decode_plan_create(opattn_plan **plan, const int
                                                    const int32_t *cu_seqlens_k, int32_t n_seq, int32_t Hq,
                                                    int32_t Hkv, int32_t d, int32_t max_ctas);
 /*
+ * Paged K/V caches (the layout of paged-attention serving engines).  k_cache
+ * and v_cache are device arrays [num_blocks, block_size, Hkv, d] bf16;
+ * sequence s owns Lk_s = seqlens_k[s] keys (HOST array of n_seq int32), and
+ * key j of s is row j % block_size of page block_table[s * max_blocks +
+ * j / block_size] (block_table: DEVICE int32 [n_seq, max_blocks], read by
+ * the kernel).  Everything else (q, o, lse, cu_seqlens_q, mask, outputs) is
+ * as for opattn_decode.  block_size must be 8, 16, 32, 64 or 128, and every
+ * sequence needs ceil(Lk_s / block_size) <= max_blocks; otherwise
+ * OPATTN_ERR_UNSUPPORTED / OPATTN_ERR_INVALID_ARG before any device work.
+ * Page ids are not checked on the host: an id outside [0, num_blocks)
+ * makes the kernel read zeros for that page, never memory outside the
+ * caches.  The rows of a sequence's last page past its last key are read
+ * and weighted by zero, so they must hold finite values (any data a reused
+ * page held before is fine; NaN or infinity there would reach O).
+ */
+OPATTN_API opattn_status opattn_decode_paged(const void *q, const void *k_cache, const void *v_cache,
+                                             const int32_t *block_table, int64_t num_blocks, int32_t block_size,
+                                             int32_t max_blocks, void *o, float *lse,
+                                             const int32_t *cu_seqlens_q, const int32_t *seqlens_k, int32_t n_seq,
+                                             int32_t Hq, int32_t Hkv, int32_t d, float scale, void *stream);
+/* A paged decode plan: built from the host key counts, run with
+ * opattn_plan_run_paged (opattn_plan_run rejects it with
+ * OPATTN_ERR_INVALID_ARG, and opattn_plan_run_paged rejects other plans). */
+OPATTN_API opattn_status opattn_decode_paged_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
+                                                         const int32_t *seqlens_k, int32_t n_seq, int32_t Hq,
+                                                         int32_t Hkv, int32_t d, int32_t block_size,
+                                                         int32_t max_blocks, int32_t max_ctas);
+OPATTN_API opattn_status opattn_plan_run_paged(const opattn_plan *plan, const void *q, const void *k_cache,
+                                               const void *v_cache, const int32_t *block_table,
+                                               int64_t num_blocks, void *o, float *lse, float scale,
+                                               void *stream);
+/*
  * Host-only decode scheduler (no GPU needed).  A unit is (sequence, kv head,
  * chunk of 128-key tiles); a sequence's tiles are cut into equal chunks so
  * that the CTAs get about six units each (at least 4 tiles per chunk), and

@@ -79,6 +79,13 @@ def load():
             lib.opattn_decode_checked.argtypes = [P, P, P, P, P, P, P, i32, i32, i32, i32, f32, P, u32]
             lib.opattn_decode_plan_create.restype = ctypes.c_int
             lib.opattn_decode_plan_create.argtypes = [ctypes.POINTER(P), P, P, i32, i32, i32, i32, i32]
+            lib.opattn_decode_paged.restype = ctypes.c_int
+            lib.opattn_decode_paged.argtypes = [P, P, P, P, i64, i32, i32, P, P, P, P, i32, i32, i32, i32, f32, P]
+            lib.opattn_decode_paged_plan_create.restype = ctypes.c_int
+            lib.opattn_decode_paged_plan_create.argtypes = [ctypes.POINTER(P), P, P, i32, i32, i32, i32, i32, i32,
+                                                            i32]
+            lib.opattn_plan_run_paged.restype = ctypes.c_int
+            lib.opattn_plan_run_paged.argtypes = [P, P, P, P, P, i64, P, P, f32, P]
             lib.opattn_decode_schedule.restype = ctypes.c_int
             lib.opattn_decode_schedule.argtypes = [P, P, i32, i32, i32, i32, i32, P, i64, P,
                                                    ctypes.POINTER(i64), ctypes.POINTER(i32)]
@@ -209,6 +216,21 @@ def opattn_decode_checked(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: in
                                             _stream_handle(stream), int(flags)))
 
 
+def opattn_decode_paged(q, k_cache, v_cache, block_table, num_blocks: int, block_size: int, max_blocks: int, o, lse,
+                        cu_seqlens_q, seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int, scale: float, stream=None,
+                        *, check: bool = True) -> int:
+    """C ``opattn_decode_paged``: decode over paged K/V caches [num_blocks, block_size, Hkv, d]
+    with a device block table [n_seq, max_blocks] and host key counts ``seqlens_k``."""
+    cq, lk = _cu(cu_seqlens_q), _cu(seqlens_k)
+    st = load().opattn_decode_paged(_dptr(q), _dptr(k_cache), _dptr(v_cache), _dptr(block_table), int(num_blocks),
+                                    int(block_size), int(max_blocks), _dptr(o), _dptr(lse), _np_ptr(cq),
+                                    _np_ptr(lk), int(n_seq), int(Hq), int(Hkv), int(d), float(scale),
+                                    _stream_handle(stream))
+    if check and st != OPATTN_OK:
+        raise OpattnError(st, "opattn_decode_paged")
+    return st
+
+
 class Plan:
     """C ``opattn_plan_*``: a work list built and uploaded once, run many times.
 
@@ -217,15 +239,23 @@ class Plan:
     """
 
     def __init__(self, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, max_ctas: int = 0,
-                 decode: bool = False):
+                 decode: bool = False, block_size: int = 0, max_blocks: int = 0):
         lib = load()
         cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
         self._h = ctypes.c_void_p()
-        self.decode = decode
-        create = lib.opattn_decode_plan_create if decode else lib.opattn_plan_create
-        st = create(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1, Hq, Hkv, d, max_ctas)
+        self.decode = decode or block_size > 0
+        self.paged = block_size > 0
+        if self.paged:
+            # paged plans take per-sequence key counts in place of cu_seqlens_k
+            name = "opattn_decode_paged_plan_create"
+            st = lib.opattn_decode_paged_plan_create(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1,
+                                                     Hq, Hkv, d, block_size, max_blocks, max_ctas)
+        else:
+            name = "opattn_decode_plan_create" if decode else "opattn_plan_create"
+            create = lib.opattn_decode_plan_create if decode else lib.opattn_plan_create
+            st = create(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1, Hq, Hkv, d, max_ctas)
         if st != OPATTN_OK:
-            raise OpattnError(st, "opattn_decode_plan_create" if decode else "opattn_plan_create")
+            raise OpattnError(st, name)
         n_units, n_ctas = ctypes.c_int64(0), ctypes.c_int32(0)
         lib.opattn_plan_info(self._h, ctypes.byref(n_units), ctypes.byref(n_ctas))
         self.n_units, self.n_ctas = n_units.value, n_ctas.value
@@ -235,6 +265,12 @@ class Plan:
                                     _stream_handle(stream))
         if st != OPATTN_OK:
             raise OpattnError(st, "opattn_plan_run")
+
+    def run_paged(self, q, k_cache, v_cache, block_table, num_blocks: int, o, lse, scale: float, stream=None) -> None:
+        st = load().opattn_plan_run_paged(self._h, _dptr(q), _dptr(k_cache), _dptr(v_cache), _dptr(block_table),
+                                          int(num_blocks), _dptr(o), _dptr(lse), float(scale), _stream_handle(stream))
+        if st != OPATTN_OK:
+            raise OpattnError(st, "opattn_plan_run_paged")
 
     def close(self) -> None:
         if self._h:

@@ -121,22 +121,35 @@ struct DParams {
     float* part_lse;
     int32_t* status;
     uint32_t flags;
+    const int32_t* block_table;  // nullptr: packed K/V
+    int32_t max_blocks;
+    int32_t page_shift;          // log2(block_size)
 };
 
-// TMA producers.  One thread loads the unit's Q^T and its K tiles, another
-// its V tiles, so that K loads run ahead as far as the K ring allows and are
-// never held behind a V slot (V(j) is freed only by PV(j), K(j) already by
-// S(j)).
+// TMA producers (whole warps).  One warp loads the unit's Q^T and its K
+// tiles, another its V tiles, so that K loads run ahead as far as the K ring
+// allows and are never held behind a V slot (V(j) is freed only by PV(j),
+// K(j) already by S(j)).  With packed K/V lane 0 issues a tile as two boxes
+// of 128 rows.  With a paged cache lane i fetches the tile's i-th page id
+// from the block table and issues that page's boxes; pages past the
+// sequence's last page repeat the last page (their keys are masked), so a
+// tile always moves kSlotBytes.
 template <bool kIsV>
 __device__ __forceinline__ void dec_producer(const CUtensorMap* tmQ, const CUtensorMap* tmKV, const DParams& p,
                                              int ubeg, int uend, uint32_t sQ, uint32_t sRing, uint32_t sBar,
-                                             volatile int32_t* abort_flag) {
+                                             int lane, volatile int32_t* abort_flag) {
     using C = DCfg;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    auto wait = [&](int b, uint32_t parity) {
+        return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
+    };
     constexpr int kSlots = kIsV ? C::kVSlots : C::kKSlots;
     constexpr int kFull = kIsV ? C::kBarVFull : C::kBarKFull;
     constexpr int kEmpty = kIsV ? C::kBarVEmpty : C::kBarKEmpty;
     const uint64_t once = ptx::policy_evict_first();  // every K/V byte is read once
+    const bool paged = p.block_table != nullptr;
+    const int page_rows = 1 << p.page_shift;
+    const int pages_per_tile = paged ? kTile >> p.page_shift : 0;
     uint32_t slot = 0, par = 0, issued = 0, items = 0;
     uint32_t q_issued[2] = {0u, 0u};
     bool aborted = false;
@@ -145,37 +158,54 @@ __device__ __forceinline__ void dec_producer(const CUtensorMap* tmQ, const CUten
         if (u.n_tiles <= 0) continue;
         if (!kIsV) {
             const int qb = static_cast<int>(items & 1u);
-            if (!bounded_wait(bar(C::kBarQEmpty + qb), (q_issued[qb] & 1u) ^ 1u, abort_flag, p.status,
-                              kWaitLimitNs)) {
+            if (!wait(C::kBarQEmpty + qb, (q_issued[qb] & 1u) ^ 1u)) {
                 aborted = true;
                 break;
             }
-            ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + qb), C::kQBytes);
+            if (lane == 0) {
+                ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + qb), C::kQBytes);
 #pragma unroll
-            for (int b = 0; b < 2; ++b)
-                ptx::tma_load_3d(sQ + qb * C::kQBytes + b * (NC * 128), tmQ, bar(C::kBarQFull + qb), b * 64,
-                                 u.kvh * p.G, u.q_tok0);
+                for (int b = 0; b < 2; ++b)
+                    ptx::tma_load_3d(sQ + qb * C::kQBytes + b * (NC * 128), tmQ, bar(C::kBarQFull + qb), b * 64,
+                                     u.kvh * p.G, u.q_tok0);
+            }
             ++q_issued[qb];
             ++items;
         }
+        const int last_page = paged ? (u.Lk - 1) >> p.page_shift : 0;
+        const int32_t* table = paged ? p.block_table + static_cast<int64_t>(u.seq) * p.max_blocks : nullptr;
         for (int j = 0; j < u.n_tiles; ++j) {
-            const int row = u.k_row0 + (u.tile0 + j) * kTile;
-            if (!bounded_wait(bar(kEmpty + slot), par ^ 1u, abort_flag, p.status, kWaitLimitNs)) {
+            if (!wait(kEmpty + slot, par ^ 1u)) {
                 aborted = true;
                 break;
             }
-            ptx::mbar_arrive_expect_tx(bar(kFull + slot), C::kSlotBytes);
+            const uint32_t dst = sRing + slot * C::kSlotBytes;
+            if (lane == 0) ptx::mbar_arrive_expect_tx(bar(kFull + slot), C::kSlotBytes);
+            __syncwarp();
+            if (!paged) {
+                if (lane == 0) {
+                    const int row = u.k_row0 + (u.tile0 + j) * kTile;
 #pragma unroll
-            for (int b = 0; b < 2; ++b)
-                ptx::tma_load_3d_hint(sRing + slot * C::kSlotBytes + b * (kTile * 128), tmKV, bar(kFull + slot),
-                                      b * 64, u.kvh, row, once);
+                    for (int b = 0; b < 2; ++b)
+                        ptx::tma_load_3d_hint(dst + b * (kTile * 128), tmKV, bar(kFull + slot), b * 64, u.kvh, row,
+                                              once);
+                }
+            } else if (lane < pages_per_tile) {
+                const int page_idx = min(((u.tile0 + j) * kTile >> p.page_shift) + lane, last_page);
+                // A bad page id only moves the box out of the cache, where TMA reads zeros.
+                const int row = static_cast<int>(static_cast<uint32_t>(table[page_idx]) << p.page_shift);
+#pragma unroll
+                for (int b = 0; b < 2; ++b)
+                    ptx::tma_load_3d_hint(dst + b * (kTile * 128) + lane * (page_rows * 128), tmKV, bar(kFull + slot),
+                                          b * 64, u.kvh, row, once);
+            }
             ++issued;
             if (++slot == kSlots) { slot = 0; par ^= 1u; }
         }
     }
-    if (aborted) {
+    if (aborted && lane == 0) {
         // Let every copy still in flight land before the CTA exits: at most
-        // one outstanding load per slot and per Q buffer (the latest).
+        // one outstanding tile per slot and per Q buffer (the latest).
         for (uint32_t s = 0; s < static_cast<uint32_t>(kSlots); ++s)
             if (issued > s) {
                 const uint32_t uses = (issued - s + kSlots - 1) / kSlots;
@@ -185,6 +215,7 @@ __device__ __forceinline__ void dec_producer(const CUtensorMap* tmQ, const CUten
             for (int i = 0; i < 2; ++i)
                 if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
     }
+    __syncwarp();
 }
 
 __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sQ,
@@ -593,11 +624,9 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
     if (warp < 8) {
         dec_softmax<NCOL>(p, ubeg, uend, tmem, sP, sRed, sBar, warp >> 2, tid & 127, abort_flag);
     } else if (warp == kWarpProducerDec) {
-        if (lane == 0) dec_producer<false>(&tmQ, &tmK, p, ubeg, uend, sQ, sK, sBar, abort_flag);
-        __syncwarp();
+        dec_producer<false>(&tmQ, &tmK, p, ubeg, uend, sQ, sK, sBar, lane, abort_flag);
     } else if (warp == kWarpProducerVDec) {
-        if (lane == 0) dec_producer<true>(&tmQ, &tmV, p, ubeg, uend, sQ, sV, sBar, abort_flag);
-        __syncwarp();
+        dec_producer<true>(&tmQ, &tmV, p, ubeg, uend, sQ, sV, sBar, lane, abort_flag);
     } else if (warp == kWarpMmaDec) {
         dec_mma(p, ubeg, uend, tmem, sQ, sK, sV, sP, sBar, abort_flag);
     }
@@ -642,12 +671,23 @@ int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream) {
     int g_shift = 0;
     while ((1 << g_shift) < G) ++g_shift;
     CUtensorMap tq, tk, tv;
-    const void* kb = a.total_k > 0 ? a.k : a.q;
-    const void* vb = a.total_k > 0 ? a.v : a.q;
-    const uint64_t krows = a.total_k > 0 ? static_cast<uint64_t>(a.total_k) : 1;
+    const bool paged = a.block_table != nullptr;
+    int page_shift = 0;
+    if (paged) {
+        while ((1 << page_shift) < a.block_size) ++page_shift;
+        if ((1 << page_shift) != a.block_size || a.block_size < 8 || a.block_size > kTile) return -5;
+    }
+    // With no keys at all no unit visits a key tile; the K/V maps then only
+    // need to be well formed, so they describe one row of q.
+    const uint64_t cache_rows = paged ? static_cast<uint64_t>(a.num_blocks) * static_cast<uint64_t>(a.block_size)
+                                      : static_cast<uint64_t>(a.total_k);
+    const void* kb = cache_rows > 0 ? a.k : a.q;
+    const void* vb = cache_rows > 0 ? a.v : a.q;
+    const uint64_t krows = cache_rows > 0 ? cache_rows : 1;
+    const uint32_t box_rows = paged ? static_cast<uint32_t>(a.block_size) : static_cast<uint32_t>(kTile);
     if (!encode_3d(fn, &tq, a.q, D, a.Hq, a.total_q, G, NC / G)) return -2;
-    if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, kTile)) return -3;
-    if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, kTile)) return -4;
+    if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, box_rows)) return -3;
+    if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, box_rows)) return -4;
     DParams kp;
     kp.units = a.units;
     kp.cta_off = a.cta_off;
@@ -662,6 +702,9 @@ int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream) {
     kp.part_lse = a.part_lse;
     kp.status = a.status;
     kp.flags = a.flags;
+    kp.block_table = a.block_table;
+    kp.max_blocks = a.max_blocks;
+    kp.page_shift = page_shift;
     // columns per softmax warpgroup
     if (a.max_cols <= 8) return launch_ncol<4>(a, tq, tk, tv, kp, stream);
     if (a.max_cols <= 16) return launch_ncol<8>(a, tq, tk, tv, kp, stream);

@@ -111,6 +111,13 @@ struct DecodeLaunchArgs {
     float* part_lse;          // device, [parts][kDecCols] (log2 domain)
     int32_t* status;          // device
     uint32_t flags;
+    // Paged K/V (block_table != nullptr): k and v are [num_blocks, block_size,
+    // Hkv, d] caches and key j of sequence s lives in page
+    // block_table[s * max_blocks + j / block_size], row j % block_size.
+    const int32_t* block_table;  // device, [n_seq][max_blocks]
+    int32_t max_blocks;
+    int32_t block_size;          // 8, 16, 32, 64 or 128
+    int64_t num_blocks;
 };
 
 // Implemented in opattn_kernel.cu.  Returns a cudaError_t (as int) or a

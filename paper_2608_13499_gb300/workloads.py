@@ -116,6 +116,7 @@ class Workload:
     input_scale: float = 1.0
     seed: int = 0
     scale: float = field(default=0.0)
+    page_size: int = 0  # > 0: the decode workload keeps K/V in a paged cache of this page size
 
     def __post_init__(self):
         if self.scale == 0.0:
@@ -225,8 +226,59 @@ def decode_spec4_llama3_70b(seed: int = 0) -> Workload:
     return Workload("decode_spec4_llama3_70b_32x16384", [4] * 32, [16384] * 32, 64, 8, 128, 1.0, seed)
 
 
+def decode_llama3_70b_paged16(seed: int = 0) -> Workload:
+    """decode_llama3_70b with its K/V in a paged cache of 16-key pages in shuffled order."""
+    w = Workload("decode_llama3_70b_paged16_64x8192", [1] * 64, [8192] * 64, 64, 8, 128, 1.0, seed)
+    w.page_size = 16
+    return w
+
+
 DECODE = {"decode_llama3_70b": decode_llama3_70b, "decode_llama3_8b": decode_llama3_8b,
-          "decode_spec4_llama3_70b": decode_spec4_llama3_70b}
+          "decode_spec4_llama3_70b": decode_spec4_llama3_70b, "decode_llama3_70b_paged16": decode_llama3_70b_paged16}
+
+
+# --------------------------------------------------------------------------
+# Paged K/V caches
+# --------------------------------------------------------------------------
+
+@dataclass
+class PagedLayout:
+    """Where each sequence's keys live in a paged cache [num_blocks, page_size, heads, d]."""
+    page_size: int
+    num_blocks: int
+    block_table: np.ndarray  # int32 [n_seq, max_blocks]; -1 where a sequence has no page
+    max_blocks: int
+
+
+def paged_layout(k_lens, page_size: int, seed: int = 0, spare: float = 0.25) -> PagedLayout:
+    """Give every sequence ceil(Lk / page_size) pages drawn in a seeded random order from a pool
+    with `spare` unused pages, so that consecutive pages of a sequence are scattered."""
+    n_pages = [(int(L) + page_size - 1) // page_size for L in k_lens]
+    total = sum(n_pages)
+    num_blocks = max(1, total + int(spare * total) + 1)
+    perm = np.random.default_rng(seed).permutation(num_blocks).astype(np.int32)
+    max_blocks = max([1] + n_pages)
+    table = np.full((len(k_lens), max_blocks), -1, dtype=np.int32)
+    off = 0
+    for s, n in enumerate(n_pages):
+        table[s, :n] = perm[off:off + n]
+        off += n
+    return PagedLayout(page_size, num_blocks, table, max_blocks)
+
+
+def to_paged(x: torch.Tensor, k_lens, layout: PagedLayout, fill: float = 7.0) -> torch.Tensor:
+    """Scatter packed rows x [total_k, heads, d] into a paged cache; every other row holds `fill`."""
+    heads, d = x.shape[1], x.shape[2]
+    cache = torch.full((layout.num_blocks, layout.page_size, heads, d), fill, dtype=x.dtype, device=x.device)
+    flat = cache.view(layout.num_blocks * layout.page_size, heads, d)
+    rows = []
+    for s, L in enumerate(k_lens):
+        j = np.arange(int(L), dtype=np.int64)
+        rows.append(layout.block_table[s, j // layout.page_size].astype(np.int64) * layout.page_size
+                    + j % layout.page_size)
+    idx = torch.from_numpy(np.concatenate(rows) if rows else np.zeros(0, dtype=np.int64)).to(x.device)
+    flat[idx] = x
+    return cache
 
 STANDARD = {"tiny": tiny, "llama3_8b": llama3_8b, "llama3_70b": llama3_70b,
             "bursty": bursty, "chunked": chunked}

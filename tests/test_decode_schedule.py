@@ -133,3 +133,30 @@ def test_decode_plan_and_schedule_validate():
     assert st == pkg.OPATTN_ERR_INVALID_ARG                             # n_ctas must be positive
     assert pkg.opattn_decode_checked(A, A, A, A, A, (0, 1), (0, 9), 1, 16, 2, 128, 0.1, stream=0,
                                      flags=0x40) == pkg.OPATTN_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(block_size=12), pkg.OPATTN_ERR_UNSUPPORTED),
+    (dict(block_size=4), pkg.OPATTN_ERR_UNSUPPORTED),
+    (dict(block_size=256), pkg.OPATTN_ERR_UNSUPPORTED),
+    (dict(max_blocks=1), pkg.OPATTN_ERR_INVALID_ARG),          # 9 keys need 2 pages of 8
+    (dict(max_blocks=0), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(seqlens_k=(-1,)), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(d=64), pkg.OPATTN_ERR_UNSUPPORTED),
+    (dict(k=None), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(table=None), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(num_blocks=0), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(table=A + 2), pkg.OPATTN_ERR_MISALIGNED),
+    (dict(v=A + 8), pkg.OPATTN_ERR_MISALIGNED),
+    (dict(seqlens_k=(0,), q=None), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(cu_q=(0, 0)), pkg.OPATTN_OK),                         # no query rows: nothing to do
+])
+def test_paged_argument_errors(kwargs, status):
+    args = dict(q=A, k=A, v=A, table=A, num_blocks=4, block_size=8, max_blocks=2, o=A, lse=A, cu_q=(0, 1),
+                seqlens_k=(9,), Hq=16, Hkv=2, d=128, scale=0.125)
+    args.update(kwargs)
+    st = pkg.opattn_decode_paged(args["q"], args["k"], args["v"], args["table"], args["num_blocks"],
+                                 args["block_size"], args["max_blocks"], args["o"], args["lse"], args["cu_q"],
+                                 args["seqlens_k"], 1, args["Hq"], args["Hkv"], args["d"], args["scale"], stream=0,
+                                 check=False)
+    assert st == status

@@ -51,3 +51,25 @@ def test_make_inputs_shapes_and_input_scale():
     assert q.dtype == torch.bfloat16
     full = W.normal_bf16(3, W.STREAM_Q, 8 * 4 * 64, "cpu", 1.0)
     assert torch.equal(q.flatten(), (full.float() * 0.5).to(torch.bfloat16))
+
+
+def test_paged_layout_round_trip():
+    """Every key row lands in its own page slot; gathering through the block table restores the packed rows."""
+    import torch
+    lens = [5, 0, 40, 17, 128, 129]
+    for page in (8, 16, 64, 128):
+        lay = W.paged_layout(lens, page, seed=3)
+        n_pages = [(L + page - 1) // page for L in lens]
+        assert lay.max_blocks == max(n_pages) and lay.block_table.shape == (len(lens), lay.max_blocks)
+        used = np.concatenate([lay.block_table[s, :n] for s, n in enumerate(n_pages)])
+        assert len(set(used.tolist())) == len(used) == sum(n_pages)       # no page shared
+        assert used.min() >= 0 and used.max() < lay.num_blocks
+        assert lay.num_blocks > sum(n_pages)                               # spare pages exist
+        for s, n in enumerate(n_pages):
+            assert np.all(lay.block_table[s, n:] == -1)
+        x = torch.arange(sum(lens) * 2 * 3, dtype=torch.float32).view(sum(lens), 2, 3)
+        cache = W.to_paged(x, lens, lay, fill=-5.0)
+        assert cache.shape == (lay.num_blocks, page, 2, 3)
+        rows = [cache[lay.block_table[s, j // page], j % page] for s, L in enumerate(lens) for j in range(L)]
+        assert torch.equal(torch.stack(rows), x)
+        assert int((cache == -5.0).all(dim=-1).all(dim=-1).sum()) == lay.num_blocks * page - sum(lens)
