@@ -180,9 +180,10 @@ OPATTN_API opattn_status opattn_schedule(const int32_t *cu_seqlens_q, const int3
  * (a few with speculative tokens) over the sequence's whole cached key
  * range.  opattn_decode computes exactly what opattn_prefill computes, with
  * the same arguments, layouts, mask and outputs, with a kernel built for
- * that shape: it is bound by reading K and V from HBM, cuts long key ranges
- * into chunks processed in parallel (split-KV) and merges the chunks'
- * partial results with their log-sum-exp weights inside the same launch.
+ * that shape: it is bound by reading K and V from HBM, cuts the key ranges
+ * into chunks processed in parallel (split-KV, balanced over the SMs) and
+ * merges the chunks' partial results with their log-sum-exp weights inside
+ * the same launch.
  *
  * Supported shapes: d = 128, G = Hq / Hkv dividing 32 (1, 2, 4, 8, 16, 32),
  * and Lq * G <= 32 for every sequence (e.g. G = 8: up to 4 query tokens per
@@ -246,9 +247,11 @@ OPATTN_API opattn_status opattn_plan_run_paged(const opattn_plan *plan, const vo
                                                void *stream);
 /*
  * Host-only decode scheduler (no GPU needed).  A unit is (sequence, kv head,
- * chunk of 128-key tiles); a sequence's tiles are cut into equal chunks so
- * that the CTAs get about six units each (at least 4 tiles per chunk), and
- * units are packed onto CTAs longest first as in opattn_schedule.  Writes
+ * range of 128-key tiles).  The tiles of all (sequence, kv head) pairs, in
+ * order, are cut into min(n_ctas, tiles) equal stretches, one per CTA, so
+ * every CTA streams the same number of tiles to within one; a pair cut by
+ * stretch boundaries becomes several chunks on consecutive CTAs.  Pairs
+ * without keys become zero-tile units spread over the CTAs.  Writes
  * `units` as 12 int32 per unit:
  *     {first packed query row, query tokens of the sequence, first packed key
  *      row, Lk, kv head, first key tile of the chunk, tiles in the chunk,

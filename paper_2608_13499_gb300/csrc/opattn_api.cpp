@@ -366,67 +366,101 @@ struct DecodeSchedule {
     int32_t n_cta = 0;
     int32_t n_groups = 0;          // split (sequence, kv head) pairs: one merge counter each
     int32_t n_parts = 0;           // partial (O, LSE) slots
-    int32_t chunk_tiles = 0;       // target key tiles per chunk
+    int32_t chunk_tiles = 0;       // key tiles per CTA (rounded up)
     int32_t max_cols = 0;          // largest G * Lq over the batch
 };
 
-constexpr int32_t kDecMinChunkTiles = 4;  // 512 keys: below this a chunk's fixed costs dominate
-constexpr int32_t kDecChunksPerCta = 6;   // aim for about this many units per CTA
-
-// Units are (sequence, kv head, chunk of key tiles).  A sequence's key tiles
-// are cut into equal chunks of about chunk_tiles tiles, with chunk_tiles
-// sized so that the CTAs get about kDecChunksPerCta units each; the units
-// are packed onto CTAs longest first (cost = tiles + 1).
+// Units are (sequence, kv head, range of key tiles).  The key tiles of all
+// (sequence, kv head) pairs, taken in order, are cut into n_cta equal
+// stretches, one per CTA (stream-K style): every CTA streams the same number
+// of tiles to within one, and a pair whose tiles fall into several
+// stretches is split into chunks there, merged later by the last chunk to
+// finish.  Pairs with no keys become zero-tile units spread over the CTAs.
 void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas,
                            DecodeSchedule* out) {
+    struct Pair {
+        int32_t s, h, n_t;
+    };
+    std::vector<Pair> pairs;
     int64_t total_tiles = 0;
-    for (int32_t s = 0; s < g.n_seq; ++s)
-        if (cu_q[s + 1] > cu_q[s]) total_tiles += static_cast<int64_t>((cu_k[s + 1] - cu_k[s] + kBlockN - 1) / kBlockN) * g.Hkv;
-    const int64_t ctas = std::max<int32_t>(max_ctas, 1);
-    const int64_t per_cta = (total_tiles + ctas - 1) / ctas;
-    const int32_t chunk = static_cast<int32_t>(
-        std::max<int64_t>(kDecMinChunkTiles, (per_cta + kDecChunksPerCta - 1) / kDecChunksPerCta));
-    std::vector<DecUnit> all;
-    int32_t max_cost = 0, n_groups = 0, n_parts = 0;
     for (int32_t s = 0; s < g.n_seq; ++s) {
-        const int32_t Lq = cu_q[s + 1] - cu_q[s];
-        if (Lq == 0) continue;
-        const int32_t Lk = cu_k[s + 1] - cu_k[s];
-        const int32_t n_t = (Lk + kBlockN - 1) / kBlockN;
-        const int32_t n_chunks = n_t == 0 ? 1 : (n_t + chunk - 1) / chunk;
-        for (int32_t h = 0; h < g.Hkv; ++h) {
-            const int32_t group = n_chunks > 1 ? n_groups++ : -1;
-            const int32_t part0 = n_chunks > 1 ? n_parts : -1;
-            if (n_chunks > 1) n_parts += n_chunks;
-            for (int32_t c = 0; c < n_chunks; ++c) {
-                const int32_t t0 = static_cast<int32_t>(static_cast<int64_t>(c) * n_t / n_chunks);
-                const int32_t t1 = static_cast<int32_t>(static_cast<int64_t>(c + 1) * n_t / n_chunks);
-                DecUnit u;
-                u.q_tok0 = cu_q[s];
-                u.nq = Lq;
-                u.k_row0 = cu_k[s];
-                u.Lk = Lk;
-                u.kvh = h;
-                u.tile0 = t0;
-                u.n_tiles = t1 - t0;
-                u.part = n_chunks > 1 ? part0 + c : -1;
-                u.group = group;
-                u.chunk = c;
-                u.n_chunks = n_chunks;
-                u.seq = s;
-                max_cost = std::max(max_cost, u.n_tiles + 1);
-                all.push_back(u);
-            }
-        }
+        if (cu_q[s + 1] == cu_q[s]) continue;
+        const int32_t n_t = (cu_k[s + 1] - cu_k[s] + kBlockN - 1) / kBlockN;
+        for (int32_t h = 0; h < g.Hkv; ++h) pairs.push_back({s, h, n_t});
+        total_tiles += static_cast<int64_t>(n_t) * g.Hkv;
     }
-    lpt_pack(all, max_cost, max_ctas, [](const DecUnit& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
-             &out->n_cta);
-    out->n_groups = n_groups;
-    out->n_parts = n_parts;
-    out->chunk_tiles = chunk;
+    out->units.clear();
+    out->cta_off.clear();
+    out->n_cta = 0;
+    out->n_groups = 0;
+    out->n_parts = 0;
     int32_t max_cols = 1;
     for (int32_t s = 0; s < g.n_seq; ++s) max_cols = std::max(max_cols, (cu_q[s + 1] - cu_q[s]) * g.G);
     out->max_cols = max_cols;
+    if (pairs.empty()) return;
+    const int32_t n_cta = static_cast<int32_t>(std::max<int64_t>(
+        1, std::min<int64_t>(std::max<int32_t>(max_ctas, 1), std::max<int64_t>(total_tiles, 1))));
+    auto bound = [&](int64_t c) { return c * total_tiles / n_cta; };  // first tile of CTA c's stretch
+    auto make = [&](const Pair& pr, int32_t t0, int32_t n) {
+        DecUnit u;
+        u.q_tok0 = cu_q[pr.s];
+        u.nq = cu_q[pr.s + 1] - cu_q[pr.s];
+        u.k_row0 = cu_k[pr.s];
+        u.Lk = cu_k[pr.s + 1] - cu_k[pr.s];
+        u.kvh = pr.h;
+        u.tile0 = t0;
+        u.n_tiles = n;
+        u.part = -1;
+        u.group = -1;
+        u.chunk = 0;
+        u.n_chunks = 1;
+        u.seq = pr.s;
+        return u;
+    };
+    std::vector<std::vector<DecUnit>> per_cta(static_cast<size_t>(n_cta));
+    int64_t pos = 0;  // global index of the pair's first tile
+    int32_t zero_rr = 0;
+    for (const Pair& pr : pairs) {
+        if (pr.n_t == 0) {
+            per_cta[static_cast<size_t>(zero_rr)].push_back(make(pr, 0, 0));
+            zero_rr = (zero_rr + 1) % n_cta;
+            continue;
+        }
+        // CTAs whose stretch meets [pos, pos + n_t)
+        int64_t c = std::min<int64_t>(n_cta - 1, pos * n_cta / total_tiles);
+        while (c > 0 && bound(c) > pos) --c;
+        while (c + 1 < n_cta && bound(c + 1) <= pos) ++c;
+        std::vector<std::pair<int64_t, DecUnit>> pieces;
+        int64_t t = pos;
+        const int64_t end = pos + pr.n_t;
+        while (t < end) {
+            const int64_t stop = std::min<int64_t>(end, bound(c + 1));
+            if (stop > t) pieces.push_back({c, make(pr, static_cast<int32_t>(t - pos), static_cast<int32_t>(stop - t))});
+            t = stop;
+            ++c;
+        }
+        const int32_t n_chunks = static_cast<int32_t>(pieces.size());
+        const int32_t group = n_chunks > 1 ? out->n_groups++ : -1;
+        const int32_t part0 = n_chunks > 1 ? out->n_parts : -1;
+        if (n_chunks > 1) out->n_parts += n_chunks;
+        for (int32_t i = 0; i < n_chunks; ++i) {
+            DecUnit& u = pieces[static_cast<size_t>(i)].second;
+            u.chunk = i;
+            u.n_chunks = n_chunks;
+            u.group = group;
+            u.part = n_chunks > 1 ? part0 + i : -1;
+            per_cta[static_cast<size_t>(pieces[static_cast<size_t>(i)].first)].push_back(u);
+        }
+        pos = end;
+    }
+    out->cta_off.assign(static_cast<size_t>(n_cta) + 1, 0);
+    for (int32_t c = 0; c < n_cta; ++c) {
+        out->cta_off[static_cast<size_t>(c) + 1] =
+            out->cta_off[static_cast<size_t>(c)] + static_cast<int32_t>(per_cta[static_cast<size_t>(c)].size());
+        out->units.insert(out->units.end(), per_cta[static_cast<size_t>(c)].begin(), per_cta[static_cast<size_t>(c)].end());
+    }
+    out->n_cta = n_cta;
+    out->chunk_tiles = static_cast<int32_t>((total_tiles + n_cta - 1) / n_cta);
 }
 
 // Device work area: [cta_off | pad 32 | units | counters (2 per group: one per

@@ -399,6 +399,21 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
             continue;
         }
         const int lim0 = u.Lk - u.nq;  // column c sees keys 0 .. lim0 + c / G
+        if (col0 >= ncols) {
+            // No column of this unit is ours: keep the P arrivals in step.
+            // Waiting for PV(g - 2) keeps an arrival from landing in the
+            // previous phase of P buffer b.
+            for (int j = 0; j < u.n_tiles; ++j) {
+                const uint32_t b = g & 1u;
+                const bool ok = g < 2u || warp_wait(C::kBarPVDone + static_cast<int>(b), ((g - 2u) >> 1) & 1u);
+                if (!ptx::bar_red_and(kBarWG, kWGThreads, ok)) return;
+                ptx::mbar_arrive(bar(C::kBarPFull + static_cast<int>(b)));
+                ++g;
+                if (++sbuf == C::kSBufs) { sbuf = 0; spar ^= 1u; }
+            }
+            continue;
+        }
+        const bool all_used = col0 + NCOL <= ncols;
         float base[NCOL], l[NCOL], lh[NCOL];
 #pragma unroll
         for (int c = 0; c < NCOL; ++c) {
@@ -411,26 +426,48 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
             // S(g) ready, and P buffer b free (last read by PV(g - 2)).
             bool ok = warp_wait(C::kBarSFull + static_cast<int>(sbuf), spar);
             if (ok && g >= 2u) ok = warp_wait(C::kBarPVDone + static_cast<int>(b), ((g - 2u) >> 1) & 1u);
-            float s[NCOL];
+            // Fast path: past the chunk's first tile (bases set), every key
+            // of the tile visible to every column, all columns in use.
+            const bool fast = j > 0 && all_used && (u.tile0 + j + 1) * kTile - 1 <= lim0;
+            uint32_t sr[NCOL];
+            float x[NCOL];  // exponent s - base per column (-inf where masked)
+            float s[NCOL];  // scaled scores, -inf where masked (slow path and rebase)
             bool need = j == 0;
             if (ok) {
                 ptx::tc_fence_after();
-                uint32_t sr[NCOL];
                 ptx::tmem_ld_n<NCOL>(tS + 32u * sbuf, sr);
                 ptx::tmem_wait_ld();
                 ptx::tmem_ld_fence<NCOL>(sr);
-                const int key = (u.tile0 + j) * kTile + tid;
+                if (fast) {
+                    const uint64_t cc = ptx::f32x2(cl, cl);
+                    float xm = -INFINITY;
 #pragma unroll
-                for (int c = 0; c < NCOL; ++c) {
-                    const bool vis = col0 + c < ncols && key <= lim0 + ((col0 + c) >> gs);
-                    s[c] = vis ? __uint_as_float(sr[c]) * cl : -INFINITY;
-                    need |= s[c] - base[c] > kRebaseSlack;
+                    for (int c = 0; c < NCOL; c += 2) {
+                        ptx::f32x2_split(ptx::fma_f32x2(ptx::f32x2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])),
+                                                        cc, ptx::f32x2(-base[c], -base[c + 1])),
+                                         x[c], x[c + 1]);
+                        xm = ptx::max3f(xm, x[c], x[c + 1]);
+                    }
+                    need = xm > kRebaseSlack;
+                } else {
+                    const int key = (u.tile0 + j) * kTile + tid;
+#pragma unroll
+                    for (int c = 0; c < NCOL; ++c) {
+                        const bool vis = col0 + c < ncols && key <= lim0 + ((col0 + c) >> gs);
+                        s[c] = vis ? __uint_as_float(sr[c]) * cl : -INFINITY;
+                        need |= s[c] - base[c] > kRebaseSlack;
+                    }
                 }
             }
             // One warpgroup barrier per tile in the common case: it carries
             // both "some column needs a new base" and "some wait failed".
-            if (ptx::bar_red_or(kBarWG, kWGThreads, need || !ok)) {
+            const bool rebase = ptx::bar_red_or(kBarWG, kWGThreads, need || !ok);
+            if (rebase) {
                 if (!ptx::bar_red_and(kBarWG, kWGThreads, ok)) return;
+                if (fast) {
+#pragma unroll
+                    for (int c = 0; c < NCOL; ++c) s[c] = __uint_as_float(sr[c]) * cl;
+                }
                 float tmax[NCOL];
                 wg_reduce<NCOL, true>(s, tmax, red_ptr(), warp, lane, kBarWG);
                 bool scaled = false;
@@ -461,20 +498,17 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
                     ptx::tmem_wait_st();
                 }
             }
-            uint32_t pk[NCOL];
+            if (rebase || !fast) {
 #pragma unroll
-            for (int c = 0; c < NCOL; ++c) {
-                const float pv = ptx::ex2_approx(s[c] - (base[c] == -INFINITY ? 0.f : base[c]));
-                pk[c] = ptx::pack_bf16x2(pv, 0.f) & 0xFFFFu;
-                l[c] += pv;
-                lh[c] += ptx::bf16lo_to_f32(pk[c]);
+                for (int c = 0; c < NCOL; ++c) x[c] = s[c] - (base[c] == -INFINITY ? 0.f : base[c]);
             }
-            // P^T stores as 32-bit words of two adjacent keys: the even lane of
-            // a pair writes column c, the odd lane column c ^ kPair, each after
-            // one exchange.  With kPair = 4 the two rows a warp writes land in
-            // opposite halves of the banks (the swizzle moves row c's chunks
-            // by c mod 8), so a warp stores 128 bytes with no conflict.
-            // Masked columns hold p = 0, so all NCOL columns are written.
+            // Probabilities two columns (c, c ^ kPair) at a time, packed into
+            // one bf16x2 word, and the P^T stores as 32-bit words of two
+            // adjacent keys: after one exchange the even lane of a pair
+            // writes column c, the odd lane column c ^ kPair.  With kPair = 4
+            // the two rows a warp writes land in opposite halves of the
+            // banks (the swizzle moves row c's chunks by c mod 8), so a warp
+            // stores 128 bytes with no conflict.  Masked columns hold p = 0.
             constexpr int kPair = NCOL >= 8 ? 4 : 1;
             const bool odd = (lane & 1) != 0;
             const uint32_t prow = sP + b * C::kPBytes + p_pair;
@@ -482,9 +516,16 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
             for (int c = 0; c < NCOL; ++c) {
                 if (c & kPair) continue;
                 const int c2 = c | kPair;
-                const uint32_t recv = __shfl_xor_sync(0xFFFFFFFFu, odd ? pk[c] : pk[c2], 1);
+                const float p0 = ptx::ex2_approx(x[c]);
+                const float p1 = ptx::ex2_approx(x[c2]);
+                const uint32_t pk = ptx::pack_bf16x2(p0, p1);  // column c low, column c2 high
+                l[c] += p0;
+                l[c2] += p1;
+                lh[c] = ptx::add_bf16lo(lh[c], pk);
+                lh[c2] = ptx::add_bf16hi(lh[c2], pk);
+                const uint32_t recv = __shfl_xor_sync(0xFFFFFFFFu, pk, 1);
+                const uint32_t word = odd ? __byte_perm(pk, recv, 0x3276) : __byte_perm(pk, recv, 0x5410);
                 const int cw = odd ? c2 : c;  // column this lane writes
-                const uint32_t word = odd ? (recv | (pk[c2] << 16)) : (pk[c] | (recv << 16));
                 ptx::st_shared_u32(prow + cw * 128 + ((p_chunk ^ ((col0 + cw) & 7)) << 4), word);
             }
             ptx::fence_proxy_async_smem();
