@@ -145,6 +145,11 @@ def attention_key(Hq: int, Hkv: int, d: int) -> OperatorKey:
     return OperatorKey("opattn_prefill", (int(Hq), int(Hkv), int(d)))
 
 
+def decode_key(Hq: int, Hkv: int, d: int) -> OperatorKey:
+    """The decode-attention operator (one query token per request over its cached keys)."""
+    return OperatorKey("opattn_decode", (int(Hq), int(Hkv), int(d)))
+
+
 def gemm_key(k_in: int, n_out: int) -> OperatorKey:
     """A token-wise projection: [tokens, k_in] x [k_in, n_out]."""
     return OperatorKey("gemm", (int(k_in), int(n_out)))
@@ -195,19 +200,22 @@ class ProfileStore:
 # ---------------------------------------------------------------- GPU side
 
 class _Buffers:
-    """Device inputs sized for the largest point; every point uses a prefix."""
+    """Device inputs sized for the largest point; every point uses a prefix.
 
-    def __init__(self, max_tokens: int, Hq: int, Hkv: int, d: int, device="cuda"):
+    ``max_queries`` query rows (default: as many as keys) and ``max_keys`` key rows.
+    """
+
+    def __init__(self, max_keys: int, Hq: int, Hkv: int, d: int, device="cuda", max_queries: int = 0):
         import torch
 
         from . import workloads as W
         self.Hq, self.Hkv, self.d = Hq, Hkv, d
-        n = max_tokens
-        self.q = W.normal_bf16(0, W.STREAM_Q, n * Hq * d, device).view(n, Hq, d)
+        n, nq = max_keys, max_queries or max_keys
+        self.q = W.normal_bf16(0, W.STREAM_Q, nq * Hq * d, device).view(nq, Hq, d)
         self.k = W.normal_bf16(0, W.STREAM_K, n * Hkv * d, device).view(n, Hkv, d)
         self.v = W.normal_bf16(0, W.STREAM_V, n * Hkv * d, device).view(n, Hkv, d)
-        self.o = torch.empty((n, Hq, d), dtype=torch.bfloat16, device=device)
-        self.lse = torch.empty((n, Hq), dtype=torch.float32, device=device)
+        self.o = torch.empty((nq, Hq, d), dtype=torch.bfloat16, device=device)
+        self.lse = torch.empty((nq, Hq), dtype=torch.float32, device=device)
 
 
 def time_callable_ms(fn, reps: int, warm_ms: float = 25.0, min_ms: float = 2.0) -> float:
@@ -263,7 +271,16 @@ def measure_ms(buf, B: int, L: int, max_ctas: int = 0, reps: int = 5) -> float:
         return _time_plan_ms(plan, buf.q, buf.k, buf.v, buf.o, buf.lse, buf.d ** -0.5, reps)
 
 
-def sm_budget_curve(w, ctas, reps: int = 5, device="cuda"):
+def measure_decode_ms(buf, B: int, L: int, max_ctas: int = 0, reps: int = 5) -> float:
+    """Median time (ms) of one decode launch: B requests, one query token each, L cached keys each."""
+    import paper_2608_13499_gb300 as pkg
+    cu_q = np.arange(B + 1, dtype=np.int32)
+    cu_k = cu_q * np.int32(L)
+    with pkg.Plan(cu_q, cu_k, buf.Hq, buf.Hkv, buf.d, max_ctas=max_ctas, decode=True) as plan:
+        return _time_plan_ms(plan, buf.q, buf.k, buf.v, buf.o, buf.lse, buf.d ** -0.5, reps)
+
+
+def sm_budget_curve(w, ctas, reps: int = 5, device="cuda", decode: bool = False):
     """[(n_ctas, ms)] for workload w with the persistent grid capped at each budget."""
     import torch
 
@@ -275,7 +292,7 @@ def sm_budget_curve(w, ctas, reps: int = 5, device="cuda"):
     lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device=device)
     out = []
     for n in ctas:
-        with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, max_ctas=n) as plan:
+        with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, max_ctas=n, decode=decode) as plan:
             out.append((plan.n_ctas, _time_plan_ms(plan, q, k, v, o, lse, w.scale, reps)))
     return out
 
@@ -337,19 +354,23 @@ def profile_accuracy(n_train: int, n_test: int, seed: int = 0, key: OperatorKey 
                      b_range=(1, 32), l_range=(128, 8192), s_range=None, reps: int = 5):
     """Fit a profile on n_train random points plus the box corners; error on n_test others.
 
-    With ``s_range`` (SM shares, e.g. (1/16, 1)) the profile is over (B, L, S).
+    With ``s_range`` (SM shares, e.g. (1/16, 1)) the profile is over (B, L, S).  A
+    ``decode_key`` profiles the decode operator: B requests of one query token
+    over L cached keys each.
     """
     rng = np.random.default_rng(seed)
     ranges = [b_range, l_range] + ([s_range] if s_range else [])
     integer = [True, True] + ([False] if s_range else [])
     train = sample_points(n_train, rng, ranges, integer)
     test = sample_points(n_test, rng, ranges, integer, corners=False, stratified=False)
-    buf = _Buffers(int(b_range[1] * l_range[1]), *key.shape)
+    decode = key.op == "opattn_decode"
+    buf = _Buffers(int(b_range[1] * l_range[1]), *key.shape, max_queries=int(b_range[1]) if decode else 0)
+    measure = measure_decode_ms if decode else measure_ms
     sms = n_sms()
 
     def run(p):
         ctas = ctas_for_share(p[2], sms) if s_range else 0
-        return measure_ms(buf, int(p[0]), int(p[1]), ctas, reps)
+        return measure(buf, int(p[0]), int(p[1]), ctas, reps)
 
     t_train = np.array([run(p) for p in train])
     t_test = np.array([run(p) for p in test])
@@ -384,24 +405,31 @@ def _report(args) -> str:
 
     from . import workloads as W
     sms = n_sms()
-    lines = ["# Operator profile of opattn_prefill: sparse sampling, piecewise interpolation, SM budget", "",
+    lines = ["# Operator profiles of opattn_prefill and opattn_decode: sparse sampling, piecewise "
+             "interpolation, SM budget", "",
              f"Command: `python -m paper_2608_13499_gb300.profiler --train {args.train} --test {args.test} "
              f"--train3 {args.train3} --test3 {args.test3} --seed {args.seed} --reps {args.reps} --out <file>"
              f"{' --dump <file>' if args.dump else ''}` "
              f"on one {torch.cuda.get_device_name(0)} ({sms} SMs).", "",
-             "Operator: Llama-3-8B attention heads (Hq 32, Hkv 8, d 128), B prompts of L tokens each, "
-             "B in [1, 32], L in [128, 8192], inputs N(0, 1) bf16.  Each point is the median of "
+             "Each point is the median of "
              f"{args.reps} CUDA-event samples after 25 ms of back-to-back warm-up launches; a sample times "
-             "enough back-to-back launches to span 2 ms and divides.  The paper's operator profiles: "
-             "7% mean and 15% P90 relative error.", ""]
+             "enough back-to-back launches to span 2 ms and divides.  Inputs N(0, 1) bf16.  The paper's "
+             "operator profiles: 7% mean and 15% P90 relative error.", "",
+             "Prefill operator: Llama-3-8B attention heads (Hq 32, Hkv 8, d 128), B prompts of L tokens each, "
+             "B in [1, 32], L in [128, 8192].", ""]
     acc2 = profile_accuracy(args.train, args.test, args.seed, reps=args.reps)
-    lines += _accuracy_section("Profile over (B, L) at the full GPU", acc2, args.train, 2)
+    lines += _accuracy_section("Prefill profile over (B, L) at the full GPU", acc2, args.train, 2)
     acc3 = profile_accuracy(args.train3, args.test3, args.seed + 1, s_range=(1.0 / 16, 1.0), reps=args.reps)
-    lines += _accuracy_section("Profile over (B, L, S), SM share S in [1/16, 1]", acc3, args.train3, 3)
+    lines += _accuracy_section("Prefill profile over (B, L, S), SM share S in [1/16, 1]", acc3, args.train3, 3)
+    lines += ["Decode operator: Llama-3-70B attention heads (Hq 64, Hkv 8, d 128), B requests of one query "
+              "token over L cached keys each, B in [1, 256], L in [256, 32768].", ""]
+    accd = profile_accuracy(args.train, args.test, args.seed + 2, key=decode_key(64, 8, 128), b_range=(1, 256),
+                            l_range=(256, 32768), reps=args.reps)
+    lines += _accuracy_section("Decode profile over (B, L) at the full GPU", accd, args.train, 2)
     if args.dump:
         blob = {name: {"train": a["profile"].to_dict(), "test": a["test"].tolist(),
                        "measured": a["measured"].tolist(), "remeasured": a["remeasured"].tolist()}
-                for name, a in (("BL", acc2), ("BLS", acc3))}
+                for name, a in (("BL", acc2), ("BLS", acc3), ("decode_BL", accd))}
         with open(args.dump, "w") as f:
             json.dump(blob, f)
     shares = (0.125, 0.25, 0.5, 0.75, 1.0)
@@ -410,11 +438,13 @@ def _report(args) -> str:
               "Time relative to the full GPU in parentheses; perfect scaling would be 1/share.", "",
               "| workload | " + " | ".join(f"{b} SMs ({100 * b / sms:.0f}%)" for b in budgets) + " |",
               "|---|" + "---|" * len(budgets)]
-    for name in ("llama3_8b", "llama3_70b", "bursty", "chunked"):
-        curve = sm_budget_curve(W.STANDARD[name](), budgets, reps=args.reps)
+    rows = [(W.STANDARD[n](), False) for n in ("llama3_8b", "llama3_70b", "bursty", "chunked")]
+    rows += [(W.DECODE[n](), True) for n in ("decode_llama3_70b", "decode_llama3_8b")]
+    for w, dec in rows:
+        curve = sm_budget_curve(w, budgets, reps=args.reps, decode=dec)
         base = curve[-1][1]
-        lines.append(f"| {W.STANDARD[name]().name} | "
-                     + " | ".join(f"{ms:.3f} ms ({ms / base:.2f}x)" for _, ms in curve) + " |")
+        lines.append(f"| {w.name} | " + " | ".join(f"{ms:.3f} ms ({ms / base:.2f}x)" for _, ms in curve) + " |")
+        torch.cuda.empty_cache()
     return "\n".join(lines) + "\n"
 
 

@@ -40,3 +40,14 @@ def test_small_profile_predicts_held_out_points():
     assert acc["errors"]["mean"] < 0.25, acc["errors"]
     prof = acc["profile"]
     np.testing.assert_allclose(prof.predict(prof.coords), prof.times_ms, rtol=1e-9)
+
+
+def test_small_decode_profile_and_budget():
+    acc = P.profile_accuracy(12, 8, seed=4, key=P.decode_key(64, 8, 128), b_range=(1, 64), l_range=(256, 8192),
+                             reps=3)
+    assert np.all(acc["measured"] > 0)
+    assert acc["errors"]["mean"] < 0.25, acc["errors"]
+    w = W.DECODE["decode_llama3_70b"]()
+    sms = P.n_sms()
+    curve = P.sm_budget_curve(w, [P.ctas_for_share(0.25, sms), sms], reps=3, decode=True)
+    assert curve[0][1] > curve[1][1]          # a quarter of the SMs cannot stream as fast as all of them
