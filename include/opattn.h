@@ -157,9 +157,12 @@ OPATTN_API opattn_status opattn_plan_info(const opattn_plan *plan, int64_t *n_un
  * Host-only scheduler (no GPU needed), exposed for testing and capacity
  * planning.  A work unit is (sequence, kv head, block of 2 * (128 / G)
  * query tokens).  Its cost is the number of 128-key tiles it visits after
- * whole tiles above the causal diagonal are skipped, plus one.  Units are
- * sorted by cost, longest first, and each is given to the CTA with the least
- * assigned cost so far (Graham's longest-processing-time rule).
+ * whole tiles above the causal diagonal are skipped, plus one.  The
+ * (sequence, kv head) pairs are gathered in order into groups of at most
+ * 48 MB of K/V (so that a group's K/V stays in L2); units are taken group by
+ * group, longest first within a group, and each is given to the CTA with the
+ * least assigned cost so far (greedy list scheduling: makespan within the
+ * mean load plus the largest unit).  A CTA runs its units in that order.
  * Writes `units` as 8 int32 per unit:
  *     {first packed query row, tokens in unit, first packed key row of the
  *      sequence, Lk, last visible key of the unit's first token, kv head,

@@ -76,31 +76,22 @@ struct Schedule {
     int32_t n_cta = 0;
 };
 
-// Longest-processing-time packing: units are bucket-sorted by cost, longest
-// first (stable: enumeration order within a cost), and each goes to the CTA
-// with the least cost so far (ties: lower CTA index); makespan within 4/3 of
-// optimal.  Writes the units grouped by CTA and the CSR offsets.
+// K/V bytes of the (sequence, kv head) pairs whose units run together: small
+// enough that their K/V stays in L2 (129 MB) while all their q-blocks read it.
+constexpr int64_t kL2GroupBytes = 48ll << 20;
+
+// Greedy list scheduling in the given order: each unit goes to the CTA with
+// the least cost so far (ties: lower CTA index); a CTA's units keep the
+// order.  Makespan within mean load + largest unit.
 template <class U, class CostFn>
-void lpt_pack(const std::vector<U>& all, int32_t max_cost, int32_t max_ctas, CostFn cost, std::vector<U>* units,
-              std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
-    const int64_t n = static_cast<int64_t>(all.size());
+void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std::vector<U>* units,
+               std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
+    const int64_t n = static_cast<int64_t>(ordered.size());
     units->clear();
     cta_off->clear();
     *n_cta_out = 0;
     if (n == 0) return;
     const int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(std::max<int32_t>(max_ctas, 1), n));
-
-    std::vector<int64_t> count(static_cast<size_t>(max_cost) + 2, 0);
-    for (const U& u : all) ++count[static_cast<size_t>(max_cost - cost(u))];
-    int64_t acc = 0;
-    for (auto& c : count) {
-        const int64_t t = c;
-        c = acc;
-        acc += t;
-    }
-    std::vector<int64_t> order(static_cast<size_t>(n));
-    for (int64_t i = 0; i < n; ++i) order[static_cast<size_t>(count[static_cast<size_t>(max_cost - cost(all[static_cast<size_t>(i)]))]++)] = i;
-
     using Slot = std::pair<int64_t, int32_t>;
     std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> heap;
     for (int32_t c = 0; c < n_cta; ++c) heap.push({0, c});
@@ -111,7 +102,7 @@ void lpt_pack(const std::vector<U>& all, int32_t max_cost, int32_t max_ctas, Cos
         heap.pop();
         owner[static_cast<size_t>(i)] = sl.second;
         ++per_cta[static_cast<size_t>(sl.second)];
-        sl.first += cost(all[static_cast<size_t>(order[static_cast<size_t>(i)])]);
+        sl.first += cost(ordered[static_cast<size_t>(i)]);
         heap.push(sl);
     }
     cta_off->assign(static_cast<size_t>(n_cta) + 1, 0);
@@ -121,30 +112,46 @@ void lpt_pack(const std::vector<U>& all, int32_t max_cost, int32_t max_ctas, Cos
     units->resize(static_cast<size_t>(n));
     for (int64_t i = 0; i < n; ++i) {
         const int32_t c = owner[static_cast<size_t>(i)];
-        (*units)[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = all[static_cast<size_t>(order[static_cast<size_t>(i)])];
+        (*units)[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = ordered[static_cast<size_t>(i)];
     }
     *n_cta_out = n_cta;
 }
 
 // Units are (sequence, kv head, block of 2 * TPB query tokens).  Cost is the
 // number of key tiles the block visits after whole tiles above the causal
-// diagonal are skipped, plus one for the Q load and the epilogue; units are
-// packed onto CTAs longest first.
+// diagonal are skipped, plus one for the Q load and the epilogue.  Pairs
+// (sequence, kv head) are taken in order and gathered into groups of at most
+// kL2GroupBytes of K/V; the units are assigned group by group, longest first
+// within a group, each to the CTA with the least cost so far.  A CTA runs its
+// units in that order, so at any time the CTAs work on one group and each
+// K/V tile comes from HBM about once; across the whole list the greedy
+// assignment keeps the makespan within mean load + largest unit.
 void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out) {
     const int32_t tpu = 2 * g.TPB;
     std::vector<UnitRec> all;
+    std::vector<int32_t> group_of;  // per unit
     int32_t max_cost = 0;
+    int32_t group = 0;
+    int64_t group_bytes = 0;
+    const int64_t pair_row_bytes = 2 * static_cast<int64_t>(g.d) * 2;  // K and V, bf16
     for (int32_t s = 0; s < g.n_seq; ++s) {
         const int32_t Lq = cu_q[s + 1] - cu_q[s];
         const int32_t Lk = cu_k[s + 1] - cu_k[s];
         const int32_t delta = Lk - Lq;
-        for (int32_t t0 = 0; t0 < Lq; t0 += tpu) {
-            const int32_t n_tok = std::min(tpu, Lq - t0);
-            const int32_t qlim0 = t0 + delta;
-            const int32_t last_key = std::min(qlim0 + n_tok - 1, Lk - 1);
-            const int32_t n_tiles = last_key < 0 ? 0 : last_key / kBlockN + 1;
-            max_cost = std::max(max_cost, n_tiles + 1);
-            for (int32_t h = 0; h < g.Hkv; ++h) {
+        if (Lq == 0) continue;
+        for (int32_t h = 0; h < g.Hkv; ++h) {
+            const int64_t pair_bytes = static_cast<int64_t>(Lk) * pair_row_bytes;
+            if (group_bytes > 0 && group_bytes + pair_bytes > kL2GroupBytes) {
+                ++group;
+                group_bytes = 0;
+            }
+            group_bytes += pair_bytes;
+            for (int32_t t0 = 0; t0 < Lq; t0 += tpu) {
+                const int32_t n_tok = std::min(tpu, Lq - t0);
+                const int32_t qlim0 = t0 + delta;
+                const int32_t last_key = std::min(qlim0 + n_tok - 1, Lk - 1);
+                const int32_t n_tiles = last_key < 0 ? 0 : last_key / kBlockN + 1;
+                max_cost = std::max(max_cost, n_tiles + 1);
                 UnitRec u;
                 u.q_tok0 = cu_q[s] + t0;
                 u.n_tok = n_tok;
@@ -155,11 +162,23 @@ void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g,
                 u.n_tiles = n_tiles;
                 u.seq = s;
                 all.push_back(u);
+                group_of.push_back(group);
             }
         }
     }
-    lpt_pack(all, max_cost, max_ctas, [](const UnitRec& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
-             &out->n_cta);
+    // group by group, longest first within a group (stable)
+    std::vector<int64_t> idx(all.size());
+    for (size_t i = 0; i < idx.size(); ++i) idx[i] = static_cast<int64_t>(i);
+    std::stable_sort(idx.begin(), idx.end(), [&](int64_t a, int64_t b) {
+        if (group_of[static_cast<size_t>(a)] != group_of[static_cast<size_t>(b)])
+            return group_of[static_cast<size_t>(a)] < group_of[static_cast<size_t>(b)];
+        return all[static_cast<size_t>(a)].n_tiles > all[static_cast<size_t>(b)].n_tiles;
+    });
+    std::vector<UnitRec> ordered;
+    ordered.reserve(all.size());
+    for (int64_t i : idx) ordered.push_back(all[static_cast<size_t>(i)]);
+    list_pack(ordered, max_ctas, [](const UnitRec& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
+              &out->n_cta);
 }
 
 // Device work area: [cta_off (n_cta + 1) | pad to 32 B | units | status].

@@ -1,8 +1,11 @@
-"""Host scheduler (longest-first ragged work list), checked without a GPU.
+"""Host scheduler (L2-grouped ragged work list), checked without a GPU.
 
 The unit records are checked against a brute-force enumeration of which
 (query token, key) pairs the causal mask leaves visible, and the assignment
-against the longest-processing-time rule and Graham's 4/3 bound.
+against a replay of its rule: (sequence, kv head) pairs gathered in order
+into groups of at most 48 MB of K/V, units taken group by group and longest
+first within a group, each given to the least-loaded CTA (list scheduling:
+makespan within mean load + largest unit).
 """
 import numpy as np
 import pytest
@@ -61,8 +64,32 @@ def test_units_cover_every_row_once_with_exact_tile_counts(case):
     assert np.all(covered == 1)
 
 
-@pytest.mark.parametrize("case", CASES)
-def test_longest_first_assignment(case):
+GROUP_BYTES = 48 << 20
+
+
+def expected_order(lq, lk, Hkv, d, G):
+    """(group, unit) keys in the order the scheduler assigns units."""
+    tpu = 2 * (128 // G)
+    keys, group, gbytes = [], 0, 0
+    for s in range(len(lq)):
+        if lq[s] == 0:
+            continue
+        for h in range(Hkv):
+            pb = lk[s] * 2 * d * 2
+            if gbytes > 0 and gbytes + pb > GROUP_BYTES:
+                group, gbytes = group + 1, 0
+            gbytes += pb
+            for t0 in range(0, lq[s], tpu):
+                n_tok = min(tpu, lq[s] - t0)
+                last = min(t0 + lk[s] - lq[s] + n_tok - 1, lk[s] - 1)
+                n_tiles = 0 if last < 0 else last // BN + 1
+                keys.append((group, n_tiles, s, h, t0))
+    # stable: group ascending, tiles descending
+    return sorted(keys, key=lambda k: (k[0], -k[1]))
+
+
+@pytest.mark.parametrize("case", CASES + [(W.chunked().q_lens, W.chunked().k_lens, 32, 8, 128, 152)])
+def test_group_major_list_assignment(case):
     lq, lk, Hq, Hkv, d, n_cta = case
     cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
     cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
@@ -70,20 +97,40 @@ def test_longest_first_assignment(case):
     n = len(units)
     if n == 0:
         return
+    G = Hq // Hkv
+    order = expected_order(lq, lk, Hkv, d, G)
+    assert len(order) == n
     P = len(offs) - 1
     assert P == min(n_cta, n)
     assert offs[0] == 0 and offs[-1] == n and np.all(np.diff(offs) >= 1)
+    # replay the greedy list assignment and compare unit by unit
+    import heapq
+    heap = [(0, c) for c in range(P)]
+    per_cta = [[] for _ in range(P)]
+    for grp, n_tiles, s, h, t0 in order:
+        load, c = heapq.heappop(heap)
+        per_cta[c].append((s, h, t0, n_tiles))
+        heapq.heappush(heap, (load + n_tiles + 1, c))
+    t = unit_table(units)
+    for c in range(P):
+        got = [(int(t["seq"][i]), int(t["kvh"][i]), int(t["q_tok0"][i] - cu_q[t["seq"][i]]), int(t["n_tiles"][i]))
+               for i in range(offs[c], offs[c + 1])]
+        assert got == per_cta[c], f"CTA {c}"
     cost = units[:, 6].astype(np.int64) + 1
     loads = np.array([cost[offs[c]:offs[c + 1]].sum() for c in range(P)])
-    for c in range(P):
-        seg = cost[offs[c]:offs[c + 1]]
-        assert np.all(np.diff(seg) <= 0), "a CTA's units are not longest first"
-    # Graham: LPT makespan <= (4/3 - 1/(3P)) * OPT, and OPT >= max(mean load, largest unit)
-    lower = max(cost.sum() / P, cost.max())
-    assert loads.max() <= (4.0 / 3.0) * lower + 1e-9
-    # greedy replay: each unit, in global longest-first order, went to a least-loaded CTA
-    order = np.argsort(-cost, kind="stable")
-    assert np.all(np.diff(cost[order]) <= 0)
+    assert loads.max() <= cost.sum() / P + cost.max() + 1e-9
+
+
+def test_groups_keep_each_groups_kv_within_l2():
+    """Llama-3-70B layer: 64 pairs of 2 MB K/V -> groups of 24 pairs (48 MB); every CTA's units visit
+    the groups in order, so the whole GPU works through one group's K/V at a time."""
+    w = W.llama3_70b()
+    units, offs = pkg.opattn_schedule(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, 152)
+    t = unit_table(units)
+    pair = t["seq"] * w.Hkv + t["kvh"]
+    group = pair // 24
+    for c in range(len(offs) - 1):
+        assert np.all(np.diff(group[offs[c]:offs[c + 1]]) >= 0)
 
 
 def test_capacity_error_reports_the_needed_size():
