@@ -461,11 +461,12 @@ def recorded_traffic(workload: str, decode: bool = False):
 
 
 def kernel_revision(decode: bool = False) -> str:
-    """Hash of the kernel sources: traffic counters are only valid for the kernel they were taken on."""
+    """Hash of the kernel and scheduler sources: traffic counters are only valid for the kernel and
+    the work order they were taken on."""
     import hashlib
     h = hashlib.sha1()
     for f in ("opattn_decode.cu" if decode else "opattn_kernel.cu", "device_common.cuh", "ptx.cuh",
-              "opattn_internal.h"):
+              "opattn_internal.h", "opattn_api.cpp"):
         with open(os.path.join(ROOT, "paper_2608_13499_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
