@@ -336,7 +336,7 @@ def run_ours(args, w):
     hq = q.cpu().pin_memory()
     hk = k.cpu().pin_memory()
     hv = v.cpu().pin_memory()
-    slots = 2
+    slots = 3
     ho = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for _ in range(slots)]
     hl = [torch.empty(lse.shape, dtype=lse.dtype).pin_memory() for _ in range(slots)]
     dq = [torch.empty_like(q) for _ in range(slots)]
@@ -372,7 +372,8 @@ def run_ours(args, w):
             e2e_step(i)
         stream.wait_stream(d2h_stream)
 
-    e2e_run(2)
+    # warm every buffer set and the library's pinned staging pool before timing
+    e2e_run(2 * slots)
     torch.cuda.synchronize(dev)
     if world > 1:
         dist.barrier()
@@ -428,7 +429,7 @@ def run_ours(args, w):
             "flops_per_step": flops,
             "roofline": roofline,
             "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "steps": e2e_steps, "pipelined": "two buffer sets; copies overlap the neighbouring steps"},
+                    "steps": e2e_steps, "pipelined": "three buffer sets; copies overlap the neighbouring steps"},
             "cpu_baseline": cpu_base,
             "clocks": clocks,
             "gpu_launches": args.steps,
