@@ -281,7 +281,8 @@ def run_ours(args, w):
         k, v = W.to_paged(k, w.k_lens, lay), W.to_paged(v, w.k_lens, lay)
         table = torch.from_numpy(lay.block_table).to(dev)
         seqlens_k = np.asarray(w.k_lens, dtype=np.int32)
-        plan = pkg.Plan(w.cu_q, seqlens_k, w.Hq, w.Hkv, w.d, block_size=w.page_size, max_blocks=lay.max_blocks)
+        plan = pkg.Plan(w.cu_q, seqlens_k, w.Hq, w.Hkv, w.d, decode=True, block_size=w.page_size,
+                        max_blocks=lay.max_blocks)
 
         def run_plan():
             plan.run_paged(q, k, v, table, lay.num_blocks, o, lse, w.scale, stream)

@@ -237,9 +237,21 @@ OPATTN_API opattn_status opattn_decode_paged(const void *q, const void *k_cache,
                                              int32_t max_blocks, void *o, float *lse,
                                              const int32_t *cu_seqlens_q, const int32_t *seqlens_k, int32_t n_seq,
                                              int32_t Hq, int32_t Hkv, int32_t d, float scale, void *stream);
-/* A paged decode plan: built from the host key counts, run with
- * opattn_plan_run_paged (opattn_plan_run rejects it with
+/* The prefill kernel over the same paged caches (e.g. a chunk of a prompt
+ * attending to its prefix in the cache): arguments as opattn_decode_paged,
+ * shapes as opattn_prefill (d = 64 or 128, G <= 128, any Lq). */
+OPATTN_API opattn_status opattn_prefill_paged(const void *q, const void *k_cache, const void *v_cache,
+                                              const int32_t *block_table, int64_t num_blocks, int32_t block_size,
+                                              int32_t max_blocks, void *o, float *lse,
+                                              const int32_t *cu_seqlens_q, const int32_t *seqlens_k, int32_t n_seq,
+                                              int32_t Hq, int32_t Hkv, int32_t d, float scale, void *stream);
+/* Paged plans (prefill or decode kernel): built from the host key counts,
+ * run with opattn_plan_run_paged (opattn_plan_run rejects them with
  * OPATTN_ERR_INVALID_ARG, and opattn_plan_run_paged rejects other plans). */
+OPATTN_API opattn_status opattn_prefill_paged_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
+                                                          const int32_t *seqlens_k, int32_t n_seq, int32_t Hq,
+                                                          int32_t Hkv, int32_t d, int32_t block_size,
+                                                          int32_t max_blocks, int32_t max_ctas);
 OPATTN_API opattn_status opattn_decode_paged_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
                                                          const int32_t *seqlens_k, int32_t n_seq, int32_t Hq,
                                                          int32_t Hkv, int32_t d, int32_t block_size,

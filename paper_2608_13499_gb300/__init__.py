@@ -84,6 +84,11 @@ def load():
             lib.opattn_decode_paged_plan_create.restype = ctypes.c_int
             lib.opattn_decode_paged_plan_create.argtypes = [ctypes.POINTER(P), P, P, i32, i32, i32, i32, i32, i32,
                                                             i32]
+            lib.opattn_prefill_paged.restype = ctypes.c_int
+            lib.opattn_prefill_paged.argtypes = [P, P, P, P, i64, i32, i32, P, P, P, P, i32, i32, i32, i32, f32, P]
+            lib.opattn_prefill_paged_plan_create.restype = ctypes.c_int
+            lib.opattn_prefill_paged_plan_create.argtypes = [ctypes.POINTER(P), P, P, i32, i32, i32, i32, i32, i32,
+                                                             i32]
             lib.opattn_plan_run_paged.restype = ctypes.c_int
             lib.opattn_plan_run_paged.argtypes = [P, P, P, P, P, i64, P, P, f32, P]
             lib.opattn_decode_schedule.restype = ctypes.c_int
@@ -216,6 +221,20 @@ def opattn_decode_checked(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: in
                                             _stream_handle(stream), int(flags)))
 
 
+def opattn_prefill_paged(q, k_cache, v_cache, block_table, num_blocks: int, block_size: int, max_blocks: int, o,
+                         lse, cu_seqlens_q, seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int, scale: float,
+                         stream=None, *, check: bool = True) -> int:
+    """C ``opattn_prefill_paged``: the prefill kernel over paged K/V caches."""
+    cq, lk = _cu(cu_seqlens_q), _cu(seqlens_k)
+    st = load().opattn_prefill_paged(_dptr(q), _dptr(k_cache), _dptr(v_cache), _dptr(block_table),
+                                     int(num_blocks), int(block_size), int(max_blocks), _dptr(o), _dptr(lse),
+                                     _np_ptr(cq), _np_ptr(lk), int(n_seq), int(Hq), int(Hkv), int(d), float(scale),
+                                     _stream_handle(stream))
+    if check and st != OPATTN_OK:
+        raise OpattnError(st, "opattn_prefill_paged")
+    return st
+
+
 def opattn_decode_paged(q, k_cache, v_cache, block_table, num_blocks: int, block_size: int, max_blocks: int, o, lse,
                         cu_seqlens_q, seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int, scale: float, stream=None,
                         *, check: bool = True) -> int:
@@ -234,8 +253,9 @@ def opattn_decode_paged(q, k_cache, v_cache, block_table, num_blocks: int, block
 class Plan:
     """C ``opattn_plan_*``: a work list built and uploaded once, run many times.
 
-    ``decode=True`` builds the plan with ``opattn_decode_plan_create`` (the
-    decode kernel); run, info and destroy are shared.
+    ``decode=True`` builds the plan for the decode kernel; ``block_size > 0``
+    builds a paged plan (``cu_seqlens_k`` is then the per-sequence key counts)
+    that runs with ``run_paged``.  Run, info and destroy are shared.
     """
 
     def __init__(self, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, max_ctas: int = 0,
@@ -243,13 +263,13 @@ class Plan:
         lib = load()
         cq, ck = _cu(cu_seqlens_q), _cu(cu_seqlens_k)
         self._h = ctypes.c_void_p()
-        self.decode = decode or block_size > 0
+        self.decode = decode
         self.paged = block_size > 0
         if self.paged:
             # paged plans take per-sequence key counts in place of cu_seqlens_k
-            name = "opattn_decode_paged_plan_create"
-            st = lib.opattn_decode_paged_plan_create(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1,
-                                                     Hq, Hkv, d, block_size, max_blocks, max_ctas)
+            name = "opattn_decode_paged_plan_create" if decode else "opattn_prefill_paged_plan_create"
+            st = getattr(lib, name)(ctypes.byref(self._h), _np_ptr(cq), _np_ptr(ck), len(cq) - 1, Hq, Hkv, d,
+                                    block_size, max_blocks, max_ctas)
         else:
             name = "opattn_decode_plan_create" if decode else "opattn_plan_create"
             create = lib.opattn_decode_plan_create if decode else lib.opattn_plan_create

@@ -276,15 +276,64 @@ LaunchArgs make_args(const void* q, const void* k, const void* v, void* o, float
     return a;
 }
 
+// Paged caches: the packed offsets the scheduler works on are built from the
+// per-sequence key counts; checks the paging arguments that need no device.
+struct PagedGeometry {
+    std::vector<int32_t> cu_k;
+    int32_t block_size = 0, max_blocks = 0;
+};
+opattn_status check_paged(const int32_t* seqlens_k, int32_t n_seq, int32_t block_size, int32_t max_blocks,
+                          PagedGeometry* pg) {
+    if (n_seq < 0) return OPATTN_ERR_INVALID_ARG;
+    if (n_seq > 0 && !seqlens_k) return OPATTN_ERR_INVALID_ARG;
+    if (block_size < 8 || block_size > kBlockN || (block_size & (block_size - 1)) != 0) return OPATTN_ERR_UNSUPPORTED;
+    if (max_blocks < 1) return OPATTN_ERR_INVALID_ARG;
+    pg->cu_k.assign(static_cast<size_t>(n_seq) + 1, 0);
+    int64_t acc = 0;
+    for (int32_t s = 0; s < n_seq; ++s) {
+        const int32_t lk = seqlens_k[s];
+        if (lk < 0) return OPATTN_ERR_INVALID_ARG;
+        if ((static_cast<int64_t>(lk) + block_size - 1) / block_size > max_blocks) return OPATTN_ERR_INVALID_ARG;
+        acc += lk;
+        if (acc >= (int64_t{1} << 31)) return OPATTN_ERR_UNSUPPORTED;
+        pg->cu_k[static_cast<size_t>(s) + 1] = static_cast<int32_t>(acc);
+    }
+    pg->block_size = block_size;
+    pg->max_blocks = max_blocks;
+    return OPATTN_OK;
+}
+opattn_status check_paged_tensors(const void* k_cache, const void* v_cache, const int32_t* block_table,
+                                  int64_t num_blocks, const Geometry& g, int32_t block_size) {
+    if (g.total_k == 0) return OPATTN_OK;
+    if (!k_cache || !v_cache || !block_table || num_blocks < 1) return OPATTN_ERR_INVALID_ARG;
+    if (!aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(block_table, 4)) return OPATTN_ERR_MISALIGNED;
+    if (num_blocks * block_size * static_cast<int64_t>(g.Hkv) >= (int64_t{1} << 31)) return OPATTN_ERR_UNSUPPORTED;
+    return OPATTN_OK;
+}
+
+struct PagedArgs {
+    const int32_t* block_table = nullptr;
+    int64_t num_blocks = 0;
+    int32_t block_size = 0, max_blocks = 0;
+};
+
 // One-shot path shared by opattn_prefill and opattn_prefill_checked.
 opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
                            const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
-                           cudaStream_t stream, uint32_t flags, bool checked) {
+                           cudaStream_t stream, uint32_t flags, bool checked, const PagedArgs* paged = nullptr) {
     Geometry g;
     opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
     if (st != OPATTN_OK) return st;
     if (g.total_q == 0) return OPATTN_OK;
-    st = check_tensors(q, k, v, o, lse, scale, g);
+    if (paged) {
+        Geometry gq = g;
+        gq.total_k = 0;  // k/v are checked as caches below
+        st = check_tensors(q, nullptr, nullptr, o, lse, scale, gq);
+        if (st == OPATTN_OK)
+            st = check_paged_tensors(k, v, paged->block_table, paged->num_blocks, g, paged->block_size);
+    } else {
+        st = check_tensors(q, k, v, o, lse, scale, g);
+    }
     if (st != OPATTN_OK) return st;
     const int sms = device_sm_count();
     if (sms <= 0) return OPATTN_ERR_CUDA;
@@ -306,7 +355,13 @@ opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o,
     staging_release(stg, stream);
     int32_t dev_status = 0;
     if (ok) {
-        const LaunchArgs a = make_args(q, k, v, o, lse, g, scale, static_cast<uint8_t*>(work), w, sch.n_cta, flags);
+        LaunchArgs a = make_args(q, k, v, o, lse, g, scale, static_cast<uint8_t*>(work), w, sch.n_cta, flags);
+        if (paged) {
+            a.block_table = paged->block_table;
+            a.max_blocks = paged->max_blocks;
+            a.block_size = paged->block_size;
+            a.num_blocks = paged->num_blocks;
+        }
         ok = launch_prefill(a, stream) == 0;
     }
     if (ok && checked) {
@@ -536,47 +591,6 @@ DecodeLaunchArgs make_decode_args(const void* q, const void* k, const void* v, v
     a.num_blocks = 0;
     return a;
 }
-
-// Paged caches: the packed offsets the scheduler works on are built from the
-// per-sequence key counts; checks the paging arguments that need no device.
-struct PagedGeometry {
-    std::vector<int32_t> cu_k;
-    int32_t block_size = 0, max_blocks = 0;
-};
-opattn_status check_paged(const int32_t* seqlens_k, int32_t n_seq, int32_t block_size, int32_t max_blocks,
-                          PagedGeometry* pg) {
-    if (n_seq < 0) return OPATTN_ERR_INVALID_ARG;
-    if (n_seq > 0 && !seqlens_k) return OPATTN_ERR_INVALID_ARG;
-    if (block_size < 8 || block_size > kBlockN || (block_size & (block_size - 1)) != 0) return OPATTN_ERR_UNSUPPORTED;
-    if (max_blocks < 1) return OPATTN_ERR_INVALID_ARG;
-    pg->cu_k.assign(static_cast<size_t>(n_seq) + 1, 0);
-    int64_t acc = 0;
-    for (int32_t s = 0; s < n_seq; ++s) {
-        const int32_t lk = seqlens_k[s];
-        if (lk < 0) return OPATTN_ERR_INVALID_ARG;
-        if ((static_cast<int64_t>(lk) + block_size - 1) / block_size > max_blocks) return OPATTN_ERR_INVALID_ARG;
-        acc += lk;
-        if (acc >= (int64_t{1} << 31)) return OPATTN_ERR_UNSUPPORTED;
-        pg->cu_k[static_cast<size_t>(s) + 1] = static_cast<int32_t>(acc);
-    }
-    pg->block_size = block_size;
-    pg->max_blocks = max_blocks;
-    return OPATTN_OK;
-}
-opattn_status check_paged_tensors(const void* k_cache, const void* v_cache, const int32_t* block_table,
-                                  int64_t num_blocks, const Geometry& g, int32_t block_size) {
-    if (g.total_k == 0) return OPATTN_OK;
-    if (!k_cache || !v_cache || !block_table || num_blocks < 1) return OPATTN_ERR_INVALID_ARG;
-    if (!aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(block_table, 4)) return OPATTN_ERR_MISALIGNED;
-    if (num_blocks * block_size * static_cast<int64_t>(g.Hkv) >= (int64_t{1} << 31)) return OPATTN_ERR_UNSUPPORTED;
-    return OPATTN_OK;
-}
-
-struct PagedArgs {
-    const int32_t* block_table = nullptr;
-    int64_t num_blocks = 0;
-    int32_t block_size = 0, max_blocks = 0;
-};
 
 opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
                           const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
@@ -872,6 +886,37 @@ opattn_status opattn_decode_plan_create(opattn_plan** plan, const int32_t* cu_se
     return decode_plan_create(plan, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, max_ctas, 0, 0);
 }
 
+opattn_status opattn_prefill_paged(const void* q, const void* k_cache, const void* v_cache,
+                                   const int32_t* block_table, int64_t num_blocks, int32_t block_size,
+                                   int32_t max_blocks, void* o, float* lse, const int32_t* cu_seqlens_q,
+                                   const int32_t* seqlens_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d,
+                                   float scale, void* stream) {
+    PagedGeometry pg;
+    opattn_status st = check_paged(seqlens_k, n_seq, block_size, max_blocks, &pg);
+    if (st != OPATTN_OK) return st;
+    PagedArgs pa;
+    pa.block_table = block_table;
+    pa.num_blocks = num_blocks;
+    pa.block_size = block_size;
+    pa.max_blocks = max_blocks;
+    return prefill_impl(q, k_cache, v_cache, o, lse, cu_seqlens_q, pg.cu_k.data(), n_seq, Hq, Hkv, d, scale,
+                        static_cast<cudaStream_t>(stream), 0u, false, &pa);
+}
+
+opattn_status opattn_prefill_paged_plan_create(opattn_plan** plan, const int32_t* cu_seqlens_q,
+                                               const int32_t* seqlens_k, int32_t n_seq, int32_t Hq, int32_t Hkv,
+                                               int32_t d, int32_t block_size, int32_t max_blocks, int32_t max_ctas) {
+    if (plan) *plan = nullptr;
+    PagedGeometry pg;
+    opattn_status st = check_paged(seqlens_k, n_seq, block_size, max_blocks, &pg);
+    if (st != OPATTN_OK) return st;
+    st = opattn_plan_create(plan, cu_seqlens_q, pg.cu_k.data(), n_seq, Hq, Hkv, d, max_ctas);
+    if (st != OPATTN_OK) return st;
+    (*plan)->block_size = block_size;
+    (*plan)->max_blocks = max_blocks;
+    return OPATTN_OK;
+}
+
 opattn_status opattn_decode_paged(const void* q, const void* k_cache, const void* v_cache, const int32_t* block_table,
                                   int64_t num_blocks, int32_t block_size, int32_t max_blocks, void* o, float* lse,
                                   const int32_t* cu_seqlens_q, const int32_t* seqlens_k, int32_t n_seq, int32_t Hq,
@@ -912,6 +957,14 @@ opattn_status opattn_plan_run_paged(const opattn_plan* plan, const void* q, cons
     if (st != OPATTN_OK) return st;
     uint8_t* work = static_cast<uint8_t*>(plan->work);
     const cudaStream_t st_ = static_cast<cudaStream_t>(stream);
+    if (!plan->decode) {
+        LaunchArgs a = make_args(q, k_cache, v_cache, o, lse, plan->g, scale, work, plan->w, plan->sch.n_cta, 0u);
+        a.block_table = block_table;
+        a.max_blocks = plan->max_blocks;
+        a.block_size = plan->block_size;
+        a.num_blocks = num_blocks;
+        return launch_prefill(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+    }
     if (cudaMemsetAsync(work + plan->dw.off_counters, 0, plan->dw.zero_bytes, st_) != cudaSuccess)
         return OPATTN_ERR_CUDA;
     DecodeLaunchArgs a = make_decode_args(q, k_cache, v_cache, o, lse, plan->g, scale, work, plan->dw,

@@ -54,6 +54,11 @@ struct LaunchArgs {
     int32_t n_cta;
     int32_t* status;          // device
     uint32_t flags;
+    // Paged K/V (block_table != nullptr): as in DecodeLaunchArgs.
+    const int32_t* block_table = nullptr;
+    int32_t max_blocks = 0;
+    int32_t block_size = 0;
+    int64_t num_blocks = 0;
 };
 
 // Limits of the allocation-free entry point (opattn_prefill_noalloc), whose

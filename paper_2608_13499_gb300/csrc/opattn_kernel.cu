@@ -100,6 +100,9 @@ struct KParams {
     float scale_log2;  // softmax scale * log2(e)
     int32_t* status;
     uint32_t flags;
+    const int32_t* block_table;  // nullptr: packed K/V
+    int32_t max_blocks;
+    int32_t page_shift;          // log2(page size)
 };
 
 template <int D>
@@ -165,6 +168,92 @@ __device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUten
         for (int i = 0; i < 2; ++i)
             if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
     }
+}
+
+// Producer for paged K/V caches (whole warp).  Same order and barriers as
+// run_producer; a K or V tile is page_size-row boxes, one page per lane:
+// lane i fetches the tile's i-th page id from the block table and issues
+// that page's boxes at row offset i * page_size of the slot (a multiple of 8
+// rows, so the 128-byte swizzle matches a 128-row box).  Pages past the
+// sequence's last page repeat it (those keys are masked), so a tile always
+// moves kSlotBytes; an out-of-range page id moves the box outside the cache,
+// where TMA reads zeros.
+template <int D>
+__device__ __forceinline__ void run_producer_paged(const CUtensorMap* tmQ, const CUtensorMap* tmK,
+                                                   const CUtensorMap* tmV, const KParams& p, int ubeg, int uend,
+                                                   uint32_t sQ, uint32_t sRing, uint32_t sBar, int lane,
+                                                   volatile int32_t* abort_flag) {
+    using C = Cfg<D>;
+    auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
+    auto wait = [&](int b, uint32_t parity) {
+        return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
+    };
+    const uint32_t q_tx = static_cast<uint32_t>(p.G * p.TPB) * C::kQTxBytesPerRow;
+    const uint64_t keep = ptx::policy_evict_last();
+    const uint64_t stream = ptx::policy_evict_first();
+    const int page_rows = 1 << p.page_shift;
+    const int pages_per_tile = kBlockN >> p.page_shift;
+    uint32_t slot = 0, ring_par = 0, ring_issued = 0;
+    uint32_t q_issued[2] = {0u, 0u};
+    bool aborted = false;
+    for (int ui = ubeg; ui < uend && !aborted; ++ui) {
+        const UnitRec u = p.units[ui];
+        if (u.n_tiles <= 0) continue;
+        for (int i = 0; i < 2; ++i) {
+            if (!wait(C::kBarQEmpty + i, (q_issued[i] & 1u) ^ 1u)) {
+                aborted = true;
+                break;
+            }
+            if (lane == 0) {
+                ptx::mbar_arrive_expect_tx(bar(C::kBarQFull + i), q_tx);
+#pragma unroll
+                for (int b = 0; b < C::kDBlocks; ++b)
+                    ptx::tma_load_3d_hint(sQ + i * C::kQTileBytes + b * (kRowsPerTile * 128), tmQ,
+                                          bar(C::kBarQFull + i), b * 64, u.kvh * p.G, u.q_tok0 + i * p.TPB, stream);
+            }
+            ++q_issued[i];
+        }
+        const int last_page = (u.Lk - 1) >> p.page_shift;
+        const int32_t* table = p.block_table + static_cast<int64_t>(u.seq) * p.max_blocks;
+        for (int j = 0; j < u.n_tiles && !aborted; ++j) {
+            // this lane's page of tile j (the page id is the same for K and V)
+            int row = 0;
+            if (lane < pages_per_tile) {
+                const int page_idx = min(((j * kBlockN) >> p.page_shift) + lane, last_page);
+                row = static_cast<int>(static_cast<uint32_t>(table[page_idx]) << p.page_shift);
+            }
+            for (int kv = 0; kv < 2; ++kv) {
+                if (!wait(C::kBarEmpty + slot, ring_par ^ 1u)) {
+                    aborted = true;
+                    break;
+                }
+                if (lane == 0) ptx::mbar_arrive_expect_tx(bar(C::kBarFull + slot), C::kSlotBytes);
+                __syncwarp();
+                if (lane < pages_per_tile) {
+#pragma unroll
+                    for (int b = 0; b < C::kDBlocks; ++b)
+                        ptx::tma_load_3d_hint(sRing + slot * C::kSlotBytes + b * (kBlockN * 128) + lane * (page_rows * 128),
+                                              kv ? tmV : tmK, bar(C::kBarFull + slot), b * 64, u.kvh, row, keep);
+                }
+                ++ring_issued;
+                if (++slot == C::kSlots) {
+                    slot = 0;
+                    ring_par ^= 1u;
+                }
+            }
+        }
+    }
+    if (aborted && lane == 0) {
+        for (uint32_t s = 0; s < static_cast<uint32_t>(C::kSlots); ++s) {
+            if (ring_issued > s) {
+                const uint32_t uses = (ring_issued - s + C::kSlots - 1) / C::kSlots;
+                drain_wait(bar(C::kBarFull + s), (uses - 1u) & 1u, kDrainLimitNs);
+            }
+        }
+        for (int i = 0; i < 2; ++i)
+            if (q_issued[i] > 0) drain_wait(bar(C::kBarQFull + i), (q_issued[i] - 1u) & 1u, kDrainLimitNs);
+    }
+    __syncwarp();
 }
 
 template <int D>
@@ -524,8 +613,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp < kWarpSoftmax) {
         ptx::setmaxnreg_dec<kRegsControl>();
         if (warp == kWarpProducer) {
-            if (lane == 0) run_producer<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, abort_flag);
-            __syncwarp();
+            if (p.block_table) {
+                run_producer_paged<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, lane, abort_flag);
+            } else {
+                if (lane == 0) run_producer<D>(&tmQ, &tmK, &tmV, p, ubeg, uend, sQ, sRing, sBar, abort_flag);
+                __syncwarp();
+            }
         } else if (warp == kWarpMma) {
             run_mma<D>(p, ubeg, uend, tmem, sQ, sRing, sBar, abort_flag);
         }
@@ -552,12 +645,21 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     CUtensorMap tq, tk, tv;
     // With no keys at all no unit visits a key tile; the K/V maps then only
     // need to be well formed, so they describe one row of q.
-    const void* kb = a.total_k > 0 ? a.k : a.q;
-    const void* vb = a.total_k > 0 ? a.v : a.q;
-    const uint64_t krows = a.total_k > 0 ? static_cast<uint64_t>(a.total_k) : 1;
+    const bool paged = a.block_table != nullptr;
+    int page_shift = 0;
+    if (paged) {
+        while ((1 << page_shift) < a.block_size) ++page_shift;
+        if ((1 << page_shift) != a.block_size || a.block_size < 8 || a.block_size > kBlockN) return -5;
+    }
+    const uint64_t cache_rows = paged ? static_cast<uint64_t>(a.num_blocks) * static_cast<uint64_t>(a.block_size)
+                                      : static_cast<uint64_t>(a.total_k);
+    const void* kb = cache_rows > 0 ? a.k : a.q;
+    const void* vb = cache_rows > 0 ? a.v : a.q;
+    const uint64_t krows = cache_rows > 0 ? cache_rows : 1;
+    const uint32_t box_rows = paged ? static_cast<uint32_t>(a.block_size) : static_cast<uint32_t>(kBlockN);
     if (!encode_3d(fn, &tq, a.q, D, a.Hq, a.total_q, G, TPB)) return -2;
-    if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, kBlockN)) return -3;
-    if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, kBlockN)) return -4;
+    if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, box_rows)) return -3;
+    if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, box_rows)) return -4;
 
     static std::mutex mu;
     static bool attr_done[128] = {};
@@ -595,6 +697,9 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     kp.scale_log2 = a.scale * kLog2e;
     kp.status = a.status;
     kp.flags = a.flags;
+    kp.block_table = a.block_table;
+    kp.max_blocks = a.max_blocks;
+    kp.page_shift = page_shift;
     opattn_prefill_kernel<D><<<a.n_cta, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, kp);
     return cudaGetLastError();
 }

@@ -97,7 +97,7 @@ def test_paged_plan_runs_repeatedly_and_rejects_packed_runs():
     o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
     o = torch.empty((w.total_q, w.Hq, w.d), dtype=torch.bfloat16, device="cuda")
     lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device="cuda")
-    with pkg.Plan(w.cu_q, np.asarray(w.k_lens, dtype=np.int32), w.Hq, w.Hkv, w.d, block_size=16,
+    with pkg.Plan(w.cu_q, np.asarray(w.k_lens, dtype=np.int32), w.Hq, w.Hkv, w.d, decode=True, block_size=16,
                   max_blocks=lay.max_blocks) as plan:
         assert plan.paged and plan.n_units > 2
         with pytest.raises(pkg.OpattnError):

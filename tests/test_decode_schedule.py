@@ -161,3 +161,22 @@ def test_paged_argument_errors(kwargs, status):
                                  args["seqlens_k"], 1, args["Hq"], args["Hkv"], args["d"], args["scale"], stream=0,
                                  check=False)
     assert st == status
+
+
+@pytest.mark.parametrize("kwargs,status", [
+    (dict(block_size=12), pkg.OPATTN_ERR_UNSUPPORTED),
+    (dict(max_blocks=1), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(d=96), pkg.OPATTN_ERR_UNSUPPORTED),
+    (dict(k=None), pkg.OPATTN_ERR_INVALID_ARG),
+    (dict(table=A + 2), pkg.OPATTN_ERR_MISALIGNED),
+    (dict(cu_q=(0, 0)), pkg.OPATTN_OK),
+])
+def test_paged_prefill_argument_errors(kwargs, status):
+    args = dict(q=A, k=A, v=A, table=A, num_blocks=4, block_size=8, max_blocks=2, o=A, lse=A, cu_q=(0, 5),
+                seqlens_k=(9,), Hq=16, Hkv=2, d=128, scale=0.125)
+    args.update(kwargs)
+    st = pkg.opattn_prefill_paged(args["q"], args["k"], args["v"], args["table"], args["num_blocks"],
+                                  args["block_size"], args["max_blocks"], args["o"], args["lse"], args["cu_q"],
+                                  args["seqlens_k"], 1, args["Hq"], args["Hkv"], args["d"], args["scale"],
+                                  stream=0, check=False)
+    assert st == status
