@@ -76,10 +76,12 @@ OPATTN_API int32_t opattn_version(void);
 OPATTN_API const char *opattn_status_string(int32_t status);
 
 /*
- * One-shot prefill attention (the definition above).  Builds the
- * longest-first work list on the host, copies it to stream-ordered device
- * scratch (cudaMallocAsync / cudaFreeAsync on `stream`) and launches one
- * persistent kernel over min(#SMs, #units) CTAs.  Returns OPATTN_OK with no
+ * One-shot prefill attention (the definition above).  Builds the work
+ * list on the host (L2-sized groups of (sequence, kv head) pairs, longest
+ * unit first within a group) in mapped pinned memory, then launches on
+ * `stream` a small upload kernel that reads it into stream-ordered device
+ * scratch (cudaMallocAsync / cudaFreeAsync) and one persistent kernel over
+ * min(#SMs, #units) CTAs; no copy-engine transfer.  Returns OPATTN_OK with no
  * device work when total_q == 0.  `scale` must be finite and > 0 (usually
  * 1 / sqrt(d)).  Device-side wait timeouts are not reported here; use
  * opattn_prefill_checked to observe them.

@@ -15,7 +15,7 @@ LIB = os.path.join(PKG, "libopattn.so")
 BUILD_DIR = os.path.join(PKG, "_build")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["opattn_kernel.cu", "opattn_decode.cu", "opattn_api.cpp", "opattn_noalloc.cu"]
+SOURCES = ["opattn_kernel.cu", "opattn_decode.cu", "opattn_api.cpp", "opattn_noalloc.cu", "opattn_upload.cu"]
 DEPS = ["ptx.cuh", "opattn_internal.h", "device_common.cuh"]
 
 

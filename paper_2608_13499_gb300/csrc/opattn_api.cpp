@@ -201,11 +201,14 @@ void pack_upload(const Schedule& s, const WorkLayout& w, uint8_t* dst) {
 }
 
 // ---------------------------------------------------- pinned staging pool
-// The work list goes to the device with an asynchronous copy from pinned
-// memory; a staging buffer is reused only after the event recorded behind
-// its copy has completed, so no call ever blocks on the GPU.
+// The work list is built in mapped pinned memory and read from there by the
+// upload kernel (opattn_upload.cu); a staging buffer is reused only after
+// the event recorded behind that read has completed, so no call ever blocks
+// on the GPU.  Where the memory cannot be mapped, an asynchronous copy
+// moves it instead.
 struct Staging {
     void* host = nullptr;
+    void* dev = nullptr;  // device address of the mapped buffer, or null
     size_t cap = 0;
     cudaEvent_t done = nullptr;
     bool busy = false;
@@ -227,9 +230,17 @@ Staging* staging_acquire(size_t bytes) {
     Staging* s = new Staging;
     size_t cap = 4096;
     while (cap < bytes) cap *= 2;
-    if (cudaHostAlloc(&s->host, cap, cudaHostAllocPortable) != cudaSuccess) {
-        delete s;
-        return nullptr;
+    if (cudaHostAlloc(&s->host, cap, cudaHostAllocPortable | cudaHostAllocMapped) == cudaSuccess) {
+        if (cudaHostGetDevicePointer(&s->dev, s->host, 0) != cudaSuccess) {
+            (void)cudaGetLastError();
+            s->dev = nullptr;
+        }
+    } else {
+        (void)cudaGetLastError();
+        if (cudaHostAlloc(&s->host, cap, cudaHostAllocPortable) != cudaSuccess) {
+            delete s;
+            return nullptr;
+        }
     }
     if (cudaEventCreateWithFlags(&s->done, cudaEventDisableTiming) != cudaSuccess) {
         cudaFreeHost(s->host);
@@ -245,6 +256,15 @@ void staging_release(Staging* s, cudaStream_t stream) {
     std::lock_guard<std::mutex> lk(g_stage_mu);
     cudaEventRecord(s->done, stream);
     s->busy = false;
+}
+// Moves the first `bytes` of a staged work list to `dst` and zeroes the
+// `zero_bytes` at `zero` (a multiple of 4), in stream order on `stream`.
+bool upload_staged(const Staging* s, void* dst, size_t bytes, void* zero, size_t zero_bytes, cudaStream_t stream) {
+    if (s->dev)
+        return launch_upload(s->dev, dst, bytes, static_cast<int32_t*>(zero), zero_bytes / sizeof(int32_t),
+                             stream) == 0;
+    return cudaMemcpyAsync(dst, s->host, bytes, cudaMemcpyHostToDevice, stream) == cudaSuccess &&
+           cudaMemsetAsync(zero, 0, zero_bytes, stream) == cudaSuccess;
 }
 
 int device_sm_count() {
@@ -350,8 +370,8 @@ opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o,
         staging_release(stg, stream);
         return OPATTN_ERR_CUDA;
     }
-    bool ok = cudaMemcpyAsync(work, stg->host, w.upload_bytes, cudaMemcpyHostToDevice, stream) == cudaSuccess;
-    ok = ok && cudaMemsetAsync(static_cast<uint8_t*>(work) + w.off_status, 0, sizeof(int32_t), stream) == cudaSuccess;
+    bool ok = upload_staged(stg, work, w.upload_bytes, static_cast<uint8_t*>(work) + w.off_status, sizeof(int32_t),
+                            stream);
     staging_release(stg, stream);
     int32_t dev_status = 0;
     if (ok) {
@@ -626,8 +646,7 @@ opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, 
         return OPATTN_ERR_CUDA;
     }
     uint8_t* wb = static_cast<uint8_t*>(work);
-    bool ok = cudaMemcpyAsync(wb, stg->host, w.upload_bytes, cudaMemcpyHostToDevice, stream) == cudaSuccess;
-    ok = ok && cudaMemsetAsync(wb + w.off_counters, 0, w.zero_bytes, stream) == cudaSuccess;
+    bool ok = upload_staged(stg, wb, w.upload_bytes, wb + w.off_counters, w.zero_bytes, stream);
     staging_release(stg, stream);
     int32_t dev_status = 0;
     if (ok) {

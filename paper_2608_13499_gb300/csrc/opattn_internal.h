@@ -132,5 +132,10 @@ int launch_prefill(const LaunchArgs& a, cudaStream_t stream);
 int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream);
 // Shared memory bytes the kernel needs for head dim d (0 if unsupported).
 int kernel_smem_bytes(int d);
+// Implemented in opattn_upload.cu: one small kernel on `stream` copies
+// `bytes` (a multiple of 16; src and dst 16-byte aligned) from src, which may
+// be mapped pinned host memory, to the device buffer dst, and zeroes
+// `zero_words` int32 words at `zero`.  Returns a cudaError_t as int.
+int launch_upload(const void* src, void* dst, size_t bytes, int32_t* zero, size_t zero_words, cudaStream_t stream);
 
 }  // namespace opattn
