@@ -17,6 +17,8 @@
 //   warps 8-11    the same for M-tile 1
 // TMEM (512 columns): S0 | S1 (128 fp32 columns each; P is written back into
 // the first 64 columns as packed bf16) | O0 | O1 (d columns each).
+// Shared memory: Q of both M-tiles | K/V ring | (d = 128) one 4 KB O staging
+// buffer per softmax warp (32 rows x 64 channels, written out by TMA stores).
 //
 // MMA order per key tile j (after the prologue S0(0), S1(0)):
 //   PV0(j), S0(j+1) -> commit S-ready[0] (or O-ready[0] after the last tile)
@@ -67,10 +69,14 @@ struct Cfg {
     static constexpr int kDBlocks = D / 64;                        // 128-byte swizzle column blocks
     static constexpr int kQTileBytes = kRowsPerTile * D * 2;       // one M-tile of Q
     static constexpr int kSlotBytes = kBlockN * D * 2;             // one K or V tile
-    static constexpr int kSlots = D == 128 ? 5 : 12;               // ring depth (K and V alternate)
+    static constexpr int kSlots = D == 128 ? 4 : 12;               // ring depth (K and V alternate)
     static constexpr int kQOff = 0;
     static constexpr int kRingOff = 2 * kQTileBytes;
-    static constexpr int kBarOff = kRingOff + kSlots * kSlotBytes;
+    // O staging for TMA stores (d = 128 only): per softmax warp 32 rows x 64 channels
+    static constexpr bool kTmaStoreO = D == 128;
+    static constexpr int kStageBytes = 32 * 128;
+    static constexpr int kStageOff = kRingOff + kSlots * kSlotBytes;
+    static constexpr int kBarOff = kStageOff + (kTmaStoreO ? 8 * kStageBytes : 0);
     static constexpr int kBarFull = 0;
     static constexpr int kBarEmpty = kSlots;
     static constexpr int kBarQFull = 2 * kSlots;       // + M-tile
@@ -103,6 +109,7 @@ struct KParams {
     const int32_t* block_table;  // nullptr: packed K/V
     int32_t max_blocks;
     int32_t page_shift;          // log2(page size)
+    int32_t o_tma;               // a warp's 32 rows form one TMA box of O (G divides 32, or 32 divides G)
 };
 
 template <int D>
@@ -436,9 +443,68 @@ __device__ __forceinline__ void store_zero_row(const KParams& p, int64_t row_idx
     p.lse[row_idx] = -INFINITY;
 }
 
+// Epilogue of one row: O / l -> bf16 into this warp's staging buffer and out
+// with TMA stores when all 32 rows of the warp belong to the unit (the box
+// would otherwise write rows of the next sequence) and d = 128, else with
+// predicated 16-byte stores per row.  The staging image is the 128-byte-swizzled box
+// (64 channels x the warp's 32 rows): 16-byte chunk c of row r sits at chunk
+// c ^ (r & 7), so the 32 lanes' writes of one chunk fill all 32 banks four
+// times over.
 template <int D>
-__device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sBar,
-                                            int warp, int lane, volatile int32_t* abort_flag) {
+__device__ __forceinline__ void store_o_rows(const KParams& p, const CUtensorMap* tmO, uint32_t sStage, uint32_t tO,
+                                             float inv_l, bool valid, int64_t row_idx, int lane, int32_t c_head,
+                                             int32_t c_tok) {
+    if (Cfg<D>::kTmaStoreO && p.o_tma && __all_sync(0xFFFFFFFFu, valid)) {
+#pragma unroll
+        for (int b = 0; b < D / 64; ++b) {
+            uint32_t w[32];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                uint32_t ov[32];
+                load_row<32>(tO + 64 * b + 32 * h, ov);
+#pragma unroll
+                for (int t = 0; t < 16; ++t)
+                    w[16 * h + t] =
+                        ptx::pack_bf16x2(__uint_as_float(ov[2 * t]) * inv_l, __uint_as_float(ov[2 * t + 1]) * inv_l);
+            }
+            if (lane == 0) ptx::bulk_wait_read_all();  // the previous store from this buffer has read it
+            __syncwarp();
+            const uint32_t row = sStage + static_cast<uint32_t>(lane) * 128u;
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                ptx::st_shared_v4(row + ((static_cast<uint32_t>(c) ^ (lane & 7u)) << 4), w[4 * c], w[4 * c + 1],
+                                  w[4 * c + 2], w[4 * c + 3]);
+            ptx::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                ptx::tma_store_3d(tmO, sStage, 64 * b, c_head, c_tok);
+                ptx::bulk_commit_group();
+            }
+        }
+        return;
+    }
+#pragma unroll
+    for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t ov[32];
+        load_row<32>(tO + 32 * ch, ov);
+        uint32_t w[16];
+#pragma unroll
+        for (int t = 0; t < 16; ++t)
+            w[t] = ptx::pack_bf16x2(__uint_as_float(ov[2 * t]) * inv_l, __uint_as_float(ov[2 * t + 1]) * inv_l);
+        if (valid) {
+            uint4* dst = reinterpret_cast<uint4*>(p.o + row_idx * D + ch * 32);
+            dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+            dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+            dst[2] = make_uint4(w[8], w[9], w[10], w[11]);
+            dst[3] = make_uint4(w[12], w[13], w[14], w[15]);
+        }
+    }
+}
+
+template <int D>
+__device__ __forceinline__ void softmax_units(const KParams& p, const CUtensorMap* tmO, int ubeg, int uend,
+                                              uint32_t tmem, uint32_t sBar, uint32_t sStage, int warp, int lane,
+                                              volatile int32_t* abort_flag) {
     using C = Cfg<D>;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
     const int mt = (warp - kWarpSoftmax) >> 2;  // M-tile
@@ -535,32 +601,30 @@ __device__ __forceinline__ void run_softmax(const KParams& p, int ubeg, int uend
         // used (a weighted mean of V rows); LSE uses the unrounded sum.
         const float inv_l = lh > 0.f ? 1.f / lh : 0.f;
         const float lse_v = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
-#pragma unroll
-        for (int ch = 0; ch < D / 32; ++ch) {
-            uint32_t ov[32];
-            ptx::tmem_ld32(tO + 32 * ch, ov);
-            ptx::tmem_wait_ld();
-            ptx::tmem_ld_fence<32>(ov);
-            uint32_t w[16];
-#pragma unroll
-            for (int t = 0; t < 16; ++t)
-                w[t] = ptx::pack_bf16x2(__uint_as_float(ov[2 * t]) * inv_l, __uint_as_float(ov[2 * t + 1]) * inv_l);
-            if (valid) {
-                uint4* dst = reinterpret_cast<uint4*>(p.o + row_idx * D + ch * 32);
-                dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
-                dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
-                dst[2] = make_uint4(w[8], w[9], w[10], w[11]);
-                dst[3] = make_uint4(w[12], w[13], w[14], w[15]);
-            }
-        }
+        // origin of the TMA box of this warp's 32 rows: (channel, head, token)
+        const int tok_w = mt * TPB + (quarter * 32) / G;
+        const int head_w = (quarter * 32) % G;
+        store_o_rows<D>(p, tmO, sStage, tO, inv_l, valid, row_idx, lane, u.kvh * G + head_w, u.q_tok0 + tok_w);
         if (valid) p.lse[row_idx] = lse_v;
     }
+}
+
+// Softmax warpgroup role; lane 0 lets its TMA stores finish before the CTA
+// exits, also when a wait timed out.
+template <int D>
+__device__ __forceinline__ void run_softmax(const KParams& p, const CUtensorMap* tmO, int ubeg, int uend,
+                                            uint32_t tmem, uint32_t sBar, uint32_t sStage, int warp, int lane,
+                                            volatile int32_t* abort_flag) {
+    softmax_units<D>(p, tmO, ubeg, uend, tmem, sBar, sStage, warp, lane, abort_flag);
+    if (lane == 0) ptx::bulk_wait_all();
+    __syncwarp();
 }
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     opattn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                          const __grid_constant__ CUtensorMap tmV, const KParams p) {
+                          const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                          const KParams p) {
     using C = Cfg<D>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_addr(smem_raw);
@@ -600,6 +664,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::prefetch_tmap(&tmQ);
         ptx::prefetch_tmap(&tmK);
         ptx::prefetch_tmap(&tmV);
+        ptx::prefetch_tmap(&tmO);
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -624,7 +689,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         ptx::setmaxnreg_inc<kRegsSoftmax>();
-        run_softmax<D>(p, ubeg, uend, tmem, sBar, warp, lane, abort_flag);
+        const uint32_t sStage = base + C::kStageOff + static_cast<uint32_t>(warp - kWarpSoftmax) * C::kStageBytes;
+        run_softmax<D>(p, &tmO, ubeg, uend, tmem, sBar, sStage, warp, lane, abort_flag);
     }
 
     ptx::tc_fence_before();
@@ -642,7 +708,7 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     if (!fn) return -1;
     const int G = a.Hq / a.Hkv;
     const int TPB = kRowsPerTile / G;
-    CUtensorMap tq, tk, tv;
+    CUtensorMap tq, tk, tv, to;
     // With no keys at all no unit visits a key tile; the K/V maps then only
     // need to be well formed, so they describe one row of q.
     const bool paged = a.block_table != nullptr;
@@ -660,6 +726,14 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     if (!encode_3d(fn, &tq, a.q, D, a.Hq, a.total_q, G, TPB)) return -2;
     if (!encode_3d(fn, &tk, kb, D, a.Hkv, krows, 1, box_rows)) return -3;
     if (!encode_3d(fn, &tv, vb, D, a.Hkv, krows, 1, box_rows)) return -4;
+    // O is written by each softmax warp for its 32 rows: G heads x 32 / G
+    // tokens, or 32 heads of one token when G > 32.  Other G (3, 5, 6, ...)
+    // split a warp's rows across tokens unevenly; those rows use plain stores
+    // and the map only needs to be well formed.
+    const bool o_tma = G <= 32 ? 32 % G == 0 : G % 32 == 0;
+    const uint32_t o_heads = o_tma ? static_cast<uint32_t>(G < 32 ? G : 32) : 1u;
+    const uint32_t o_tokens = o_tma ? 32u / o_heads : 1u;
+    if (!encode_3d(fn, &to, a.o, D, a.Hq, a.total_q, o_heads, o_tokens)) return -7;
 
     static std::mutex mu;
     static bool attr_done[128] = {};
@@ -700,7 +774,8 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     kp.block_table = a.block_table;
     kp.max_blocks = a.max_blocks;
     kp.page_shift = page_shift;
-    opattn_prefill_kernel<D><<<a.n_cta, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, kp);
+    kp.o_tma = o_tma ? 1 : 0;
+    opattn_prefill_kernel<D><<<a.n_cta, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, to, kp);
     return cudaGetLastError();
 }
 

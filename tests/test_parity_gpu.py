@@ -67,6 +67,13 @@ SMALL = [
     custom("g128_d64", [70, 3], [70, 3], 128, 1, 64),
     custom("long_1500_g8", [1500], [1500], 16, 2, 128, seed=3),
     custom("g2_d128_odd", [333, 1, 190], [333, 1, 190], 4, 2, 128, seed=5),
+    # d = 128 group sizes of the TMA-store epilogue (whole warps of valid rows go
+    # out as one box) and of its per-row fallback (G not dividing 32)
+    custom("g1_d128", [1, 130, 257], [1, 130, 257], 4, 4, 128, seed=6),
+    custom("g16_d128", [300, 9], [300, 9], 32, 2, 128, seed=7),
+    custom("g32_d128", [7, 64], [7, 64], 32, 1, 128, seed=8),
+    custom("g64_d128", [5, 70], [5, 70], 64, 1, 128, seed=9),
+    custom("g6_d128", [50, 200], [60, 200], 12, 2, 128, seed=10),
 ]
 
 
