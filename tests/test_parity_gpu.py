@@ -155,8 +155,10 @@ def test_full_size_workloads_sampled_rows(w):
     check(o_rows, lse_rows, o_ref, lse_ref, w.name)
 
 
-def test_outputs_stay_inside_their_buffers():
-    w = custom("canary", [130, 7], [130, 7], 8, 2, 128)
+@pytest.mark.parametrize("Hq,Hkv", [(8, 2), (32, 2), (64, 1)], ids=["g4", "g16", "g64"])
+def test_outputs_stay_inside_their_buffers(Hq, Hkv):
+    # the O epilogue writes whole warps of rows as TMA boxes: none may reach past the tensors
+    w = custom("canary", [130, 7], [130, 7], Hq, Hkv, 128)
     q, k, v = W.make_inputs(w, "cuda")
     n_o, n_l = w.total_q * w.Hq * w.d, w.total_q * w.Hq
     o_buf = torch.full((n_o + 4096,), 3.0, dtype=torch.bfloat16, device="cuda")
