@@ -203,6 +203,8 @@ def oracle_sample(w, q, k, v, seconds: float, seed: int = 0):
 
 # ----------------------------------------------------------- reference arm
 
+REFERENCE_BUDGET_S = 150.0  # host time of the reference arm's timed steps
+
 def run_reference(args, w):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -211,7 +213,9 @@ def run_reference(args, w):
     from paper_2608_13499_gb300 import workloads as W
     q, k, v = W.make_inputs(w, "cpu")
     qb, kb, vb = q, k, v
-    per_step = max(0.5, args.reference_step_seconds)
+    # Each step is a bounded sample; the whole timed run stays within about
+    # REFERENCE_BUDGET_S however many steps are asked for.
+    per_step = min(args.reference_step_seconds, max(0.05, REFERENCE_BUDGET_S / max(1, args.steps)))
     for _ in range(args.warmup):
         oracle_sample(w, qb, kb, vb, per_step / 4, seed=1)
     flops, secs, rows = 0, 0.0, 0
@@ -486,7 +490,9 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--reference-step-seconds", type=float, default=3.0)
+    ap.add_argument("--reference-step-seconds", type=float, default=3.0,
+                    help="oracle time per reference step, capped so that all steps take about "
+                         f"{REFERENCE_BUDGET_S:.0f} s")
     args = ap.parse_args(argv)
     from paper_2608_13499_gb300 import workloads as W
     w = {**W.STANDARD, **W.DECODE}[args.workload]()
