@@ -374,8 +374,12 @@ __device__ __forceinline__ void run_mma(const KParams& p, int ubeg, int uend, ui
 // N consecutive TMEM columns of this thread's lane into registers.
 template <int N>
 __device__ __forceinline__ void load_row(uint32_t taddr, uint32_t* r) {
+    if constexpr (N == 128) {
+        ptx::tmem_ld128(taddr, r);
+    } else {
 #pragma unroll
-    for (int c = 0; c < N; c += 32) ptx::tmem_ld32(taddr + c, r + c);
+        for (int c = 0; c < N; c += 32) ptx::tmem_ld32(taddr + c, r + c);
+    }
     ptx::tmem_wait_ld();
     ptx::tmem_ld_fence<N>(r);
 }
@@ -576,8 +580,7 @@ __device__ __forceinline__ void softmax_units(const KParams& p, const CUtensorMa
             }
             l = l * alpha + sum;
             lh = lh * alpha + sumh;
-            ptx::tmem_st32(tS + 0, s);
-            ptx::tmem_st32(tS + 32, s + 32);
+            ptx::tmem_st64(tS, s);
             ptx::tmem_wait_st();
             if (__any_sync(0xFFFFFFFFu, rescale)) {
 #pragma unroll
