@@ -471,7 +471,7 @@ struct DecodeSchedule {
 // stretches is split into chunks there, merged later by the last chunk to
 // finish.  Pairs with no keys become zero-tile units spread over the CTAs.
 void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas,
-                           DecodeSchedule* out) {
+                           DecodeSchedule* out, bool fit_grid = false) {
     struct Pair {
         int32_t s, h, n_t;
     };
@@ -492,6 +492,34 @@ void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geome
     for (int32_t s = 0; s < g.n_seq; ++s) max_cols = std::max(max_cols, (cu_q[s + 1] - cu_q[s]) * g.G);
     out->max_cols = max_cols;
     if (pairs.empty()) return;
+    // When every (sequence, kv head) pair has the same number of key tiles,
+    // a grid of n CTAs splits no pair if n divides the pair count, and splits
+    // every pair into equal chunks if the pair count divides n (and n / pairs
+    // divides a pair's tiles).  A split pair costs its chunks a partial write
+    // and its last chunk a merge (2-9% of such batches, measured), so with
+    // fit_grid the largest such grid down to 4/5 of max_ctas is taken.
+    if (fit_grid && max_ctas > 1) {
+        int32_t tp = -1;
+        int64_t n_pairs = 0;
+        bool uniform = true;
+        for (const Pair& pr : pairs) {
+            if (pr.n_t == 0) continue;
+            if (tp < 0) tp = pr.n_t;
+            uniform = uniform && pr.n_t == tp;
+            ++n_pairs;
+        }
+        if (uniform && n_pairs > 0) {
+            const int32_t lo = (max_ctas * 4 + 4) / 5;
+            for (int32_t n = max_ctas; n >= lo; --n) {
+                const bool whole = n_pairs % n == 0;
+                const bool equal = n % n_pairs == 0 && tp % (n / n_pairs) == 0;
+                if (whole || equal) {
+                    max_ctas = n;
+                    break;
+                }
+            }
+        }
+    }
     const int32_t n_cta = static_cast<int32_t>(std::max<int64_t>(
         1, std::min<int64_t>(std::max<int32_t>(max_ctas, 1), std::max<int64_t>(total_tiles, 1))));
     auto bound = [&](int64_t c) { return c * total_tiles / n_cta; };  // first tile of CTA c's stretch
@@ -635,7 +663,7 @@ opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, 
     if (sms <= 0) return OPATTN_ERR_CUDA;
 
     DecodeSchedule sch;
-    build_decode_schedule(cu_q, cu_k, g, sms, &sch);
+    build_decode_schedule(cu_q, cu_k, g, sms, &sch, /*fit_grid=*/true);
     const DecodeLayout w = decode_layout(sch);
     Staging* stg = staging_acquire(w.upload_bytes);
     if (!stg) return OPATTN_ERR_CUDA;
@@ -878,7 +906,9 @@ opattn_status decode_plan_create(opattn_plan** plan, const int32_t* cu_q, const 
             return OPATTN_ERR_CUDA;
         }
         const int32_t cap = max_ctas > 0 ? std::min(max_ctas, sms) : sms;
-        build_decode_schedule(cu_q, cu_k, g, cap, &p->dsch);
+        // an explicit SM budget is kept exactly; the default grid may shrink
+        // a little so that a uniform batch splits no pair
+        build_decode_schedule(cu_q, cu_k, g, cap, &p->dsch, /*fit_grid=*/max_ctas == 0);
         p->dw = decode_layout(p->dsch);
         std::vector<uint8_t> host(p->dw.upload_bytes, 0);
         pack_decode_upload(p->dsch, p->dw, host.data());

@@ -186,3 +186,23 @@ def test_full_size_workloads_on_sampled_rows(name):
     o_r, lse_r = oracle.attention_rows(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale,
                                        tok, hd)
     check(o[tok, hd], lse[tok, hd], o_r, lse_r, name)
+
+
+def test_default_grid_splits_no_pair_of_a_uniform_batch():
+    # 64 requests x 8192 keys, 8 kv heads: 512 (sequence, kv head) pairs of 64 key tiles each
+    w = W.DECODE["decode_llama3_70b"]()
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    pairs = w.n_seq * w.Hkv
+    fits = [n for n in range((sms * 4 + 4) // 5, sms + 1) if pairs % n == 0]
+    with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=True) as plan:
+        assert (sms * 4 + 4) // 5 <= plan.n_ctas <= sms
+        if fits:
+            assert plan.n_ctas == max(fits)
+            assert plan.n_units == pairs  # whole pairs per CTA: nothing split, nothing merged
+    # an explicit SM budget is kept as given
+    with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=True, max_ctas=sms) as plan:
+        assert plan.n_ctas == sms
+    # a ragged batch keeps the full grid
+    r = W.DECODE["decode_llama3_8b"]()
+    with pkg.Plan(r.cu_q, r.cu_k, r.Hq, r.Hkv, r.d, decode=True) as plan:
+        assert plan.n_ctas == sms
