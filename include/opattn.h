@@ -212,8 +212,12 @@ OPATTN_API opattn_status opattn_decode_checked(const void *q, const void *k, con
  * A plan for the decode kernel: same contract as opattn_plan_create, and the
  * plan is run, queried and destroyed with opattn_plan_run / _info / _destroy.
  * The plan owns the chunk partials, so two runs of one plan must not overlap
- * (run them on one stream).  Each run zeroes the plan's merge counters with
- * an asynchronous memset before the launch.
+ * (run them on one stream).  A run is one kernel launch and nothing else: the
+ * plan's merge counters are zeroed when it is created and every completed run
+ * leaves them at zero, so runs can also be captured in a CUDA graph and
+ * replayed.  Plan runs do not read the device status word; a run that hit a
+ * device wait timeout leaves the counters undefined, and the plan must then
+ * be destroyed rather than run again.
  */
 OPATTN_API opattn_status opattn_decode_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
                                                    const int32_t *cu_seqlens_k, int32_t n_seq, int32_t Hq,

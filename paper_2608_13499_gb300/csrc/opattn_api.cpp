@@ -588,8 +588,10 @@ void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geome
 // Device work area: [cta_off | pad 32 | units | counters (2 per group: one per
 // softmax warpgroup) | status |
 // pad 256 | part_lse (n_parts x kDecCols) | part_o (n_parts x kDecCols x d)].
-// The counters and the status word are contiguous and zeroed before every
-// launch.
+// The counters and the status word are contiguous.  One-shot calls zero them
+// with the work-list upload before every launch; a plan zeroes them once when
+// it is created, and every launch that completes leaves the counters at zero
+// (the merging chunk resets its counter), so plan runs need no memset.
 struct DecodeLayout {
     size_t off_units, off_counters, off_status, off_part_lse, off_part_o, bytes, upload_bytes, zero_bytes;
 };
@@ -808,8 +810,6 @@ opattn_status opattn_plan_run(const opattn_plan* plan, const void* q, const void
     uint8_t* work = static_cast<uint8_t*>(plan->work);
     const cudaStream_t st_ = static_cast<cudaStream_t>(stream);
     if (plan->decode) {
-        if (cudaMemsetAsync(work + plan->dw.off_counters, 0, plan->dw.zero_bytes, st_) != cudaSuccess)
-            return OPATTN_ERR_CUDA;
         const DecodeLaunchArgs a =
             make_decode_args(q, k, v, o, lse, plan->g, scale, work, plan->dw, plan->dsch.n_cta, plan->dsch.max_cols, 0u);
         return launch_decode(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
@@ -910,13 +910,15 @@ opattn_status decode_plan_create(opattn_plan** plan, const int32_t* cu_q, const 
         // a little so that a uniform batch splits no pair
         build_decode_schedule(cu_q, cu_k, g, cap, &p->dsch, /*fit_grid=*/max_ctas == 0);
         p->dw = decode_layout(p->dsch);
-        std::vector<uint8_t> host(p->dw.upload_bytes, 0);
+        // the work list, then the counters and the status word at zero
+        const size_t init_bytes = p->dw.off_counters + p->dw.zero_bytes;
+        std::vector<uint8_t> host(init_bytes, 0);
         pack_decode_upload(p->dsch, p->dw, host.data());
         if (cudaMalloc(&p->work, p->dw.bytes) != cudaSuccess) {
             delete p;
             return OPATTN_ERR_CUDA;
         }
-        if (cudaMemcpy(p->work, host.data(), p->dw.upload_bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+        if (cudaMemcpy(p->work, host.data(), init_bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
             cudaFree(p->work);
             delete p;
             return OPATTN_ERR_CUDA;
@@ -1014,8 +1016,6 @@ opattn_status opattn_plan_run_paged(const opattn_plan* plan, const void* q, cons
         a.num_blocks = num_blocks;
         return launch_prefill(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
     }
-    if (cudaMemsetAsync(work + plan->dw.off_counters, 0, plan->dw.zero_bytes, st_) != cudaSuccess)
-        return OPATTN_ERR_CUDA;
     DecodeLaunchArgs a = make_decode_args(q, k_cache, v_cache, o, lse, plan->g, scale, work, plan->dw,
                                           plan->dsch.n_cta, plan->dsch.max_cols, 0u);
     a.block_table = block_table;

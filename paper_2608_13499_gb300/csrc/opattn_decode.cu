@@ -572,17 +572,26 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
         __threadfence();
         ptx::bar_sync(kBarWG, kWGThreads);
         bool last = false;
-        // Each warpgroup counts the chunks of its own columns.
-        if (tid == 0) last = atomicAdd(p.counters + 2 * u.group + wg, 1) == u.n_chunks - 1;
+        // Each warpgroup counts the chunks of its own columns.  The chunk that
+        // finishes last has seen every arrival of this launch on its counter
+        // and sets it back to zero for the next launch of the same work list.
+        if (tid == 0) {
+            int32_t* counter = p.counters + 2 * u.group + wg;
+            last = atomicAdd(counter, 1) == u.n_chunks - 1;
+            if (last) *counter = 0;
+        }
         last = ptx::bar_red_or(kBarWG, kWGThreads, last);
         if (!last) continue;
         // This unit finished last: merge the (sequence, kv head)'s partials,
         // O = sum_k 2^(lse_k - lse) O_k with lse = log2 sum_k 2^lse_k, in one
-        // online pass over the chunks.  Each step loads every column's partial
-        // LSE and O of one chunk at once, so a chunk costs one L2 round trip
-        // rather than two per column.
+        // online pass over the chunks.  The loads of kMergeBatch chunks (every
+        // column's partial LSE and O) are issued together before any of them
+        // is used, so a batch of chunks costs one L2 round trip.  Up to 64
+        // loaded values per thread; at 16 columns one chunk's 32 already fill
+        // the registers the softmax leaves free.
         __threadfence();
         const int part0 = u.part - u.chunk;
+        constexpr int kMergeBatch = NCOL >= 16 ? 1 : 32 / NCOL;
         float m[NCOL], acc[NCOL], wsum[NCOL];
 #pragma unroll
         for (int c = 0; c < NCOL; ++c) {
@@ -590,19 +599,10 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
             acc[c] = 0.f;
             wsum[c] = 0.f;
         }
-        for (int k = 0; k < u.n_chunks; ++k) {
-            const float* plse = p.part_lse + (part0 + k) * NC + col0;
-            const float* po_k = p.part_o + (static_cast<int64_t>(part0 + k) * NC + col0) * D + tid;
-            float lk[NCOL], ok[NCOL];
+        auto merge_chunk = [&](const float (&lk)[NCOL], const float (&ok)[NCOL]) {
 #pragma unroll
             for (int c = 0; c < NCOL; ++c) {
-                const bool used = col0 + c < ncols;
-                lk[c] = used ? __ldcg(plse + c) : -INFINITY;
-                ok[c] = used ? __ldcg(po_k + c * D) : 0.f;
-            }
-#pragma unroll
-            for (int c = 0; c < NCOL; ++c) {
-                if (lk[c] == -INFINITY) continue;  // this chunk saw no key of column c
+                if (lk[c] == -INFINITY) continue;  // this chunk saw no key of column c (or is past the last)
                 const float nm = fmaxf(m[c], lk[c]);
                 const float a = m[c] == -INFINITY ? 0.f : ptx::ex2_approx(m[c] - nm);
                 const float w = ptx::ex2_approx(lk[c] - nm);
@@ -610,6 +610,39 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
                 wsum[c] = wsum[c] * a + w;
                 m[c] = nm;
             }
+        };
+        if constexpr (kMergeBatch == 1) {
+            for (int k = 0; k < u.n_chunks; ++k) {
+                const float* plse = p.part_lse + (part0 + k) * NC + col0;
+                const float* po_k = p.part_o + (static_cast<int64_t>(part0 + k) * NC + col0) * D + tid;
+                float lk[NCOL], ok[NCOL];
+#pragma unroll
+                for (int c = 0; c < NCOL; ++c) {
+                    const bool used = col0 + c < ncols;
+                    lk[c] = used ? __ldcg(plse + c) : -INFINITY;
+                    ok[c] = used ? __ldcg(po_k + c * D) : 0.f;
+                }
+                merge_chunk(lk, ok);
+            }
+        } else {
+        for (int k0 = 0; k0 < u.n_chunks; k0 += kMergeBatch) {
+            float lk[kMergeBatch][NCOL], ok[kMergeBatch][NCOL];
+#pragma unroll
+            for (int i = 0; i < kMergeBatch; ++i) {
+                const int k = k0 + i;
+                const bool have = k < u.n_chunks;
+                const float* plse = p.part_lse + static_cast<int64_t>(part0 + (have ? k : 0)) * NC + col0;
+                const float* po_k = p.part_o + (static_cast<int64_t>(part0 + (have ? k : 0)) * NC + col0) * D + tid;
+#pragma unroll
+                for (int c = 0; c < NCOL; ++c) {
+                    const bool used = have && col0 + c < ncols;
+                    lk[i][c] = used ? __ldcg(plse + c) : -INFINITY;
+                    ok[i][c] = used ? __ldcg(po_k + c * D) : 0.f;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < kMergeBatch; ++i) merge_chunk(lk[i], ok[i]);
+        }
         }
 #pragma unroll
         for (int c = 0; c < NCOL; ++c) {

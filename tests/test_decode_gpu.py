@@ -137,7 +137,7 @@ def test_matches_prefill_kernel_on_the_same_batch():
 
 
 def test_plan_repeat_runs_on_a_side_stream():
-    """A plan zeroes its merge counters before every run: repeated runs stay correct."""
+    """Each completed run leaves the plan's merge counters at zero: repeated runs stay correct."""
     w = custom("dec_plan_repeat", [1, 1], [30000, 7000], 16, 2, seed=14)
     q, k, v = W.make_inputs(w, "cuda")
     o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
@@ -153,6 +153,30 @@ def test_plan_repeat_runs_on_a_side_stream():
                 plan.run(q, k, v, o, lse, w.scale, side)
         side.synchronize()
         check(o, lse, o_ref, lse_ref, "plan x3")
+
+
+def test_plan_run_replays_from_a_cuda_graph():
+    """A decode plan run is one kernel launch that leaves its merge counters at zero, so a
+    captured run replays correctly, over key ranges split into up to 19 chunks."""
+    w = custom("dec_graph", [1, 1, 1], [6268, 512, 3000], 64, 8, seed=16)
+    q, k, v = W.make_inputs(w, "cuda")
+    o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
+    with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=True) as plan:
+        assert plan.n_units > 2 * w.Hkv * w.n_seq  # the key ranges are split
+        o = torch.empty((w.total_q, w.Hq, w.d), dtype=torch.bfloat16, device="cuda")
+        lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device="cuda")
+        plan.run(q, k, v, o, lse, w.scale)  # outside the capture: first-use set-up
+        torch.cuda.synchronize()
+        check(o, lse, o_ref, lse_ref, "eager")
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            plan.run(q, k, v, o, lse, w.scale)
+        for i in range(4):
+            o.fill_(float("nan"))
+            lse.fill_(float("nan"))
+            graph.replay()
+            torch.cuda.synchronize()
+            check(o, lse, o_ref, lse_ref, f"replay {i}")
 
 
 def test_forced_timeout_reports_and_context_survives():
