@@ -23,6 +23,8 @@ every layer, or in two models with the same head geometry) share one profile
   at ``max_ctas`` CTAs.  The kernel keeps one CTA per SM, so the cap is the
   operator's SM budget S (the paper's S_v, §3.1).
 * ``sm_budget_curve``: latency against SM share for a workload.
+* ``colocate``: two operators (prefill and decode) running at once on
+  disjoint SM budgets, against time slicing the whole GPU between them.
 * ``profile_accuracy``: relative error of an interpolated profile on
   held-out random points.  The paper's operator profiles reach 7% mean and
   15% P90 relative error (§5, "Profiling-driven Model Accuracy").
@@ -297,6 +299,78 @@ def sm_budget_curve(w, ctas, reps: int = 5, device="cuda", decode: bool = False)
     return out
 
 
+def colocate(w_a, w_b, ctas_a: int, ctas_b: int, decode_a: bool = False, decode_b: bool = True,
+             span_ms: float = 20.0, reps: int = 3, device="cuda") -> dict:
+    """Two operators sharing the GPU spatially (§2.1, "Sensitivity to SM Core Allocation").
+
+    Operator A (workload ``w_a``) runs with its persistent grid capped at
+    ``ctas_a`` CTAs on one stream, operator B at ``ctas_b`` on another; with
+    ``ctas_a + ctas_b`` at most the SM count and one CTA per SM, both grids
+    are resident at once on disjoint SMs, and neither kernel waits on the
+    other.  Each stream gets about ``span_ms`` of launches (counted from the
+    operator's time alone at its budget), all queued behind one event so
+    that they start together.  Returns the per-launch times alone (at the
+    budget and at the full GPU) and co-located, and the co-located makespan
+    against running the same launches one operator after the other on the
+    whole GPU (time slicing).
+    """
+    import torch
+
+    import paper_2608_13499_gb300 as pkg
+
+    from . import workloads as W
+    sms = n_sms()
+    if ctas_a + ctas_b > sms:
+        raise ValueError(f"budgets {ctas_a} + {ctas_b} exceed the {sms} SMs")
+
+    def operator(w, dec, n):
+        q, k, v = W.make_inputs(w, device)
+        o = torch.empty((w.total_q, w.Hq, w.d), dtype=torch.bfloat16, device=device)
+        lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device=device)
+        plan = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, max_ctas=n, decode=dec)
+        full = pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=dec)
+        return plan, full, (q, k, v, o, lse, w.scale)
+
+    plan_a, full_a, args_a = operator(w_a, decode_a, ctas_a)
+    plan_b, full_b, args_b = operator(w_b, decode_b, ctas_b)
+    try:
+        alone_a, alone_b = _time_plan_ms(plan_a, *args_a, reps), _time_plan_ms(plan_b, *args_b, reps)
+        full_ms_a, full_ms_b = _time_plan_ms(full_a, *args_a, reps), _time_plan_ms(full_b, *args_b, reps)
+        n_a = max(1, int(math.ceil(span_ms / alone_a)))
+        n_b = max(1, int(math.ceil(span_ms / alone_b)))
+        main = torch.cuda.current_stream()
+        s_a, s_b = torch.cuda.Stream(), torch.cuda.Stream()
+        samples = []
+        for _ in range(reps):
+            start = torch.cuda.Event(enable_timing=True)
+            end_a, end_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda._sleep(10_000_000)  # a few ms, so that every launch below is queued before the start
+            start.record(main)
+            s_a.wait_event(start)
+            s_b.wait_event(start)
+            for _ in range(n_a):
+                plan_a.run(*args_a, s_a)
+            end_a.record(s_a)
+            for _ in range(n_b):
+                plan_b.run(*args_b, s_b)
+            end_b.record(s_b)
+            end_a.synchronize()
+            end_b.synchronize()
+            samples.append((start.elapsed_time(end_a), start.elapsed_time(end_b)))
+        main.wait_stream(s_a)
+        main.wait_stream(s_b)
+        t_a = statistics.median(a for a, _ in samples)
+        t_b = statistics.median(b for _, b in samples)
+        makespan = statistics.median(max(a, b) for a, b in samples)
+        sliced = n_a * full_ms_a + n_b * full_ms_b
+        return {"ctas": (ctas_a, ctas_b), "launches": (n_a, n_b), "alone_ms": (alone_a, alone_b),
+                "full_gpu_ms": (full_ms_a, full_ms_b), "colocated_ms": (t_a / n_a, t_b / n_b),
+                "makespan_ms": makespan, "time_sliced_ms": sliced, "speedup": sliced / makespan}
+    finally:
+        for p in (plan_a, full_a, plan_b, full_b):
+            p.close()
+
+
 class GemmOperator:
     """Times a bf16 token-wise projection (library matmul) for B prompts of L tokens."""
 
@@ -445,7 +519,33 @@ def _report(args) -> str:
         base = curve[-1][1]
         lines.append(f"| {w.name} | " + " | ".join(f"{ms:.3f} ms ({ms / base:.2f}x)" for _, ms in curve) + " |")
         torch.cuda.empty_cache()
+    lines += [""] + _colocation_section(args.reps)
     return "\n".join(lines) + "\n"
+
+
+def _colocation_section(reps: int) -> list:
+    import torch
+
+    from . import workloads as W
+    sms = n_sms()
+    wa, wb = W.STANDARD["llama3_70b"](), W.DECODE["decode_llama3_70b"]()
+    lines = ["## Prefill and decode co-located on disjoint SM budgets", "",
+             f"Prefill: {wa.name} (one Llama-3-70B layer's attention, compute-bound); decode: {wb.name} "
+             "(HBM-bound).  Both run at once, each on its own stream with its persistent grid capped at its "
+             "budget, for about 20 ms of launches each; 'time-sliced' runs the same launches one operator after "
+             f"the other on all {sms} SMs.  Median of {reps} runs.", "",
+             "| SMs prefill + decode | prefill ms: alone at budget / co-located | decode ms: alone at budget / "
+             "co-located | makespan | time-sliced | speedup |", "|---|---|---|---|---|---|"]
+    for frac_b in (0.125, 0.25, 0.5):
+        nb = ctas_for_share(frac_b, sms)
+        r = colocate(wa, wb, sms - nb, nb, reps=reps)
+        lines.append(f"| {sms - nb} + {nb} | {r['alone_ms'][0]:.3f} / {r['colocated_ms'][0]:.3f} | "
+                     f"{r['alone_ms'][1]:.3f} / {r['colocated_ms'][1]:.3f} | {r['makespan_ms']:.1f} ms | "
+                     f"{r['time_sliced_ms']:.1f} ms | {r['speedup']:.2f}x |")
+        torch.cuda.empty_cache()
+    lines += ["", f"Alone on all {sms} SMs: prefill {r['full_gpu_ms'][0]:.3f} ms, decode "
+              f"{r['full_gpu_ms'][1]:.3f} ms per launch.", ""]
+    return lines
 
 
 def main(argv=None):
@@ -460,9 +560,14 @@ def main(argv=None):
     ap.add_argument("--dump", default=None, help="write every measured point as JSON")
     ap.add_argument("--store", default=None,
                     help="only build the Llama-3-8B layer's operator profiles and save them here as JSON")
+    ap.add_argument("--colocate", action="store_true",
+                    help="only measure prefill and decode co-located on disjoint SM budgets")
     args = ap.parse_args(argv)
     from . import build
     build.build()
+    if args.colocate:
+        print("\n".join(_colocation_section(args.reps)))
+        return
     if args.store:
         store = build_store(args.train, args.seed, reps=args.reps)
         store.save(args.store)
