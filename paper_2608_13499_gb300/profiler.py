@@ -310,9 +310,10 @@ def colocate(w_a, w_b, ctas_a: int, ctas_b: int, decode_a: bool = False, decode_
     other.  Each stream gets about ``span_ms`` of launches (counted from the
     operator's time alone at its budget), all queued behind one event so
     that they start together.  Returns the per-launch times alone (at the
-    budget and at the full GPU) and co-located, and the co-located makespan
-    against running the same launches one operator after the other on the
-    whole GPU (time slicing).
+    budget and at the full GPU) and co-located, each operator's interference
+    factor I = co-located / alone at the same SM allocation (§4.4), and the
+    co-located makespan against running the same launches one operator after
+    the other on the whole GPU (time slicing).
     """
     import torch
 
@@ -365,6 +366,7 @@ def colocate(w_a, w_b, ctas_a: int, ctas_b: int, decode_a: bool = False, decode_
         sliced = n_a * full_ms_a + n_b * full_ms_b
         return {"ctas": (ctas_a, ctas_b), "launches": (n_a, n_b), "alone_ms": (alone_a, alone_b),
                 "full_gpu_ms": (full_ms_a, full_ms_b), "colocated_ms": (t_a / n_a, t_b / n_b),
+                "interference": (t_a / n_a / alone_a, t_b / n_b / alone_b),
                 "makespan_ms": makespan, "time_sliced_ms": sliced, "speedup": sliced / makespan}
     finally:
         for p in (plan_a, full_a, plan_b, full_b):
@@ -533,14 +535,16 @@ def _colocation_section(reps: int) -> list:
              f"Prefill: {wa.name} (one Llama-3-70B layer's attention, compute-bound); decode: {wb.name} "
              "(HBM-bound).  Both run at once, each on its own stream with its persistent grid capped at its "
              "budget, for about 20 ms of launches each; 'time-sliced' runs the same launches one operator after "
-             f"the other on all {sms} SMs.  Median of {reps} runs.", "",
-             "| SMs prefill + decode | prefill ms: alone at budget / co-located | decode ms: alone at budget / "
-             "co-located | makespan | time-sliced | speedup |", "|---|---|---|---|---|---|"]
-    for frac_b in (0.125, 0.25, 0.5):
+             f"the other on all {sms} SMs.  I is the interference factor of §4.4: co-located over "
+             f"alone at the same SM allocation.  Median of {reps} runs.", "",
+             "| SMs prefill + decode | prefill ms: alone at budget / co-located (I) | decode ms: alone at budget / "
+             "co-located (I) | makespan | time-sliced | speedup |", "|---|---|---|---|---|---|"]
+    for frac_b in (0.125, 0.25, 0.375, 0.5, 0.625, 0.75):
         nb = ctas_for_share(frac_b, sms)
         r = colocate(wa, wb, sms - nb, nb, reps=reps)
-        lines.append(f"| {sms - nb} + {nb} | {r['alone_ms'][0]:.3f} / {r['colocated_ms'][0]:.3f} | "
-                     f"{r['alone_ms'][1]:.3f} / {r['colocated_ms'][1]:.3f} | {r['makespan_ms']:.1f} ms | "
+        lines.append(f"| {sms - nb} + {nb} | {r['alone_ms'][0]:.3f} / {r['colocated_ms'][0]:.3f} "
+                     f"({r['interference'][0]:.3f}) | {r['alone_ms'][1]:.3f} / {r['colocated_ms'][1]:.3f} "
+                     f"({r['interference'][1]:.3f}) | {r['makespan_ms']:.1f} ms | "
                      f"{r['time_sliced_ms']:.1f} ms | {r['speedup']:.2f}x |")
         torch.cuda.empty_cache()
     lines += ["", f"Alone on all {sms} SMs: prefill {r['full_gpu_ms'][0]:.3f} ms, decode "

@@ -64,6 +64,7 @@ def test_colocated_operators_share_the_gpu():
     assert r["ctas"] == (sms - nb, nb)
     assert all(t > 0 for t in r["alone_ms"] + r["colocated_ms"] + r["full_gpu_ms"])
     assert r["makespan_ms"] > 0 and r["speedup"] > 0
+    assert all(i > 0 for i in r["interference"])
     # outputs of co-located launches equal those of the same plans run alone
     outs = {}
     for mode in ("alone", "together"):
