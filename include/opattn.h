@@ -285,6 +285,24 @@ OPATTN_API opattn_status opattn_decode_schedule(const int32_t *cu_seqlens_q, con
                                                 int32_t n_ctas, int32_t *units, int64_t unit_capacity,
                                                 int32_t *cta_offsets, int64_t *n_units_out,
                                                 int32_t *n_ctas_used);
+/*
+ * The decode schedule that the one-shot decode calls and decode plans without
+ * an SM budget (max_ctas = 0) build on a device with `sms` SMs.  A batch whose
+ * (sequence, kv head) pairs all have the same number of key tiles takes the
+ * largest grid down to 4/5 of `sms` that splits no pair, or splits every pair
+ * into equal chunks.  A batch with at most `sms` pairs may instead be cut
+ * pair by pair: every pair into ceil(tiles / M) nearly equal chunks, one CTA
+ * each, for the smallest M that fits; that cut is taken when a cost model
+ * (a CTA's key tiles, plus five tiles' time per unit in its chain, plus two
+ * when a pair is split, with HBM saturated by about 96 streaming CTAs) rates
+ * it no slower than the stream-K cut.  Same outputs and errors as
+ * opattn_decode_schedule; `sms` must be positive.
+ */
+OPATTN_API opattn_status opattn_decode_schedule_default(const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
+                                                        int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d,
+                                                        int32_t sms, int32_t *units, int64_t unit_capacity,
+                                                        int32_t *cta_offsets, int64_t *n_units_out,
+                                                        int32_t *n_ctas_used);
 
 #ifdef __cplusplus
 }

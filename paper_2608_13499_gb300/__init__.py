@@ -94,6 +94,9 @@ def load():
             lib.opattn_decode_schedule.restype = ctypes.c_int
             lib.opattn_decode_schedule.argtypes = [P, P, i32, i32, i32, i32, i32, P, i64, P,
                                                    ctypes.POINTER(i64), ctypes.POINTER(i32)]
+            lib.opattn_decode_schedule_default.restype = ctypes.c_int
+            lib.opattn_decode_schedule_default.argtypes = [P, P, i32, i32, i32, i32, i32, P, i64, P,
+                                                           ctypes.POINTER(i64), ctypes.POINTER(i32)]
             _lib = lib
     return _lib
 
@@ -192,6 +195,13 @@ def _schedule(fn_name: str, width: int, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv
 def opattn_schedule(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):
     """C ``opattn_schedule`` (host only).  Returns (units [n, 8] int32, cta_offsets [n_ctas_used + 1])."""
     return _schedule("opattn_schedule", len(UNIT_FIELDS), cu_seqlens_q, cu_seqlens_k, Hq, Hkv, d, n_ctas)
+
+
+def opattn_decode_schedule_default(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, sms: int):
+    """C ``opattn_decode_schedule_default`` (host only): the schedule of the default decode grid on a
+    device with ``sms`` SMs.  Returns (units [n, 12] int32, cta_offsets)."""
+    return _schedule("opattn_decode_schedule_default", len(DEC_UNIT_FIELDS), cu_seqlens_q, cu_seqlens_k, Hq, Hkv,
+                     d, sms)
 
 
 def opattn_decode_schedule(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <array>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -455,7 +456,7 @@ opattn_status check_decode_geometry(const int32_t* cu_q, const Geometry& g) {
 }
 
 struct DecodeSchedule {
-    std::vector<DecUnit> units;    // grouped by CTA, longest first within a CTA
+    std::vector<DecUnit> units;    // grouped by CTA, in pair order within a CTA, then zero-tile units
     std::vector<int32_t> cta_off;  // n_cta + 1
     int32_t n_cta = 0;
     int32_t n_groups = 0;          // split (sequence, kv head) pairs: one merge counter each
@@ -464,24 +465,140 @@ struct DecodeSchedule {
     int32_t max_cols = 0;          // largest G * Lq over the batch
 };
 
-// Units are (sequence, kv head, range of key tiles).  The key tiles of all
-// (sequence, kv head) pairs, taken in order, are cut into n_cta equal
-// stretches, one per CTA (stream-K style): every CTA streams the same number
-// of tiles to within one, and a pair whose tiles fall into several
-// stretches is split into chunks there, merged later by the last chunk to
-// finish.  Pairs with no keys become zero-tile units spread over the CTAs.
+struct DecPair {
+    int32_t s, h, n_t;  // sequence, kv head, key tiles
+};
+
+// Appends pair `pr` cut into `pieces` (CTA, first tile, tiles) to the per-CTA
+// unit lists; a pair in several pieces gets a merge counter and contiguous
+// partial slots.
+void add_pair_units(const DecPair& pr, const std::vector<std::array<int64_t, 3>>& pieces, const int32_t* cu_q,
+                    const int32_t* cu_k, DecodeSchedule* out, std::vector<std::vector<DecUnit>>* per_cta) {
+    const int32_t n_chunks = static_cast<int32_t>(pieces.size());
+    const int32_t group = n_chunks > 1 ? out->n_groups++ : -1;
+    const int32_t part0 = n_chunks > 1 ? out->n_parts : -1;
+    if (n_chunks > 1) out->n_parts += n_chunks;
+    for (int32_t i = 0; i < n_chunks; ++i) {
+        DecUnit u;
+        u.q_tok0 = cu_q[pr.s];
+        u.nq = cu_q[pr.s + 1] - cu_q[pr.s];
+        u.k_row0 = cu_k[pr.s];
+        u.Lk = cu_k[pr.s + 1] - cu_k[pr.s];
+        u.kvh = pr.h;
+        u.tile0 = static_cast<int32_t>(pieces[static_cast<size_t>(i)][1]);
+        u.n_tiles = static_cast<int32_t>(pieces[static_cast<size_t>(i)][2]);
+        u.part = n_chunks > 1 ? part0 + i : -1;
+        u.group = group;
+        u.chunk = i;
+        u.n_chunks = n_chunks;
+        u.seq = pr.s;
+        (*per_cta)[static_cast<size_t>(pieces[static_cast<size_t>(i)][0])].push_back(u);
+    }
+}
+
+// Stream-K cut: the key tiles of all pairs, taken in order, are cut into
+// n_cta equal stretches, one per CTA, so every CTA streams the same number of
+// tiles to within one; a pair whose tiles fall into several stretches is
+// split into chunks there.
+void stream_k_cut(const std::vector<DecPair>& pairs, int64_t total_tiles, int32_t n_cta, const int32_t* cu_q,
+                  const int32_t* cu_k, DecodeSchedule* out, std::vector<std::vector<DecUnit>>* per_cta) {
+    auto bound = [&](int64_t c) { return c * total_tiles / n_cta; };  // first tile of CTA c's stretch
+    int64_t pos = 0;  // global index of the pair's first tile
+    for (const DecPair& pr : pairs) {
+        if (pr.n_t == 0) continue;
+        // CTAs whose stretch meets [pos, pos + n_t)
+        int64_t c = std::min<int64_t>(n_cta - 1, pos * n_cta / total_tiles);
+        while (c > 0 && bound(c) > pos) --c;
+        while (c + 1 < n_cta && bound(c + 1) <= pos) ++c;
+        std::vector<std::array<int64_t, 3>> pieces;
+        int64_t t = pos;
+        const int64_t end = pos + pr.n_t;
+        while (t < end) {
+            const int64_t stop = std::min<int64_t>(end, bound(c + 1));
+            if (stop > t) pieces.push_back({c, t - pos, stop - t});
+            t = stop;
+            ++c;
+        }
+        add_pair_units(pr, pieces, cu_q, cu_k, out, per_cta);
+        pos = end;
+    }
+}
+
+// Pair-aligned cut, for at most n_cta pairs with keys: the smallest chunk
+// size M such that sum_p ceil(t_p / M) chunks fit the grid; pair p is cut
+// into ceil(t_p / M) nearly equal chunks, one CTA each.  Every CTA then holds
+// one chunk, where a stream-K stretch can hold the end of one split pair and
+// the start of the next.  Returns the CTAs used.
+int32_t pair_aligned_cut(const std::vector<DecPair>& pairs, int32_t n_cta, const int32_t* cu_q, const int32_t* cu_k,
+                         DecodeSchedule* out, std::vector<std::vector<DecUnit>>* per_cta) {
+    int32_t hi = 1;
+    for (const DecPair& pr : pairs) hi = std::max(hi, pr.n_t);
+    auto need = [&](int32_t m) {
+        int64_t n = 0;
+        for (const DecPair& pr : pairs) n += (pr.n_t + m - 1) / m;
+        return n;
+    };
+    int32_t lo = 1;  // smallest m with need(m) <= n_cta; need(hi) = pairs with keys <= n_cta
+    while (lo < hi) {
+        const int32_t mid = lo + (hi - lo) / 2;
+        if (need(mid) <= n_cta) hi = mid; else lo = mid + 1;
+    }
+    per_cta->assign(static_cast<size_t>(need(lo)), {});
+    int64_t c = 0;
+    for (const DecPair& pr : pairs) {
+        if (pr.n_t == 0) continue;
+        const int32_t k = (pr.n_t + lo - 1) / lo;
+        std::vector<std::array<int64_t, 3>> pieces;
+        for (int32_t i = 0; i < k; ++i) {
+            const int64_t t0 = static_cast<int64_t>(pr.n_t) * i / k;
+            const int64_t t1 = static_cast<int64_t>(pr.n_t) * (i + 1) / k;
+            pieces.push_back({c++, t0, t1 - t0});
+        }
+        add_pair_units(pr, pieces, cu_q, cu_k, out, per_cta);
+    }
+    return static_cast<int32_t>(per_cta->size());
+}
+
+// Model of a decode launch's time, in key-tile times, from its per-CTA unit
+// lists (fitted to plan-run latencies of small batches on GB300: ~0.8 us per
+// key tile of a CTA's chain, ~3.8 us per extra unit in the chain; HBM is
+// saturated by about 96 CTAs streaming at once).
+double decode_schedule_cost(const std::vector<std::vector<DecUnit>>& per_cta, int64_t total_tiles) {
+    int64_t max_tiles = 0, max_units = 0;
+    bool split = false;
+    for (const auto& us : per_cta) {
+        int64_t t = 0, n = 0;
+        for (const DecUnit& u : us) {
+            if (u.n_tiles <= 0) continue;
+            t += u.n_tiles;
+            ++n;
+            split = split || u.n_chunks > 1;
+        }
+        max_tiles = std::max(max_tiles, t);
+        max_units = std::max(max_units, n);
+    }
+    return std::max(static_cast<double>(total_tiles) / 96.0, static_cast<double>(max_tiles)) + 5.0 * max_units +
+           (split ? 2.0 : 0.0);
+}
+
+// Units are (sequence, kv head, range of key tiles); a pair split into chunks
+// is merged later by the last chunk to finish.  The default cut is stream-K
+// (stream_k_cut).  With fit_grid (the default grid of a one-shot call or a
+// plan without an SM budget) a uniform batch takes a grid that splits no
+// pair, and a batch with no more pairs than CTAs takes the pair-aligned cut
+// (pair_aligned_cut) when the cost model says it is faster.  Pairs with no
+// keys become zero-tile units spread over the CTAs.
 void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas,
                            DecodeSchedule* out, bool fit_grid = false) {
-    struct Pair {
-        int32_t s, h, n_t;
-    };
-    std::vector<Pair> pairs;
+    std::vector<DecPair> pairs;
     int64_t total_tiles = 0;
+    int64_t n_pairs = 0;  // pairs with keys
     for (int32_t s = 0; s < g.n_seq; ++s) {
         if (cu_q[s + 1] == cu_q[s]) continue;
         const int32_t n_t = (cu_k[s + 1] - cu_k[s] + kBlockN - 1) / kBlockN;
         for (int32_t h = 0; h < g.Hkv; ++h) pairs.push_back({s, h, n_t});
         total_tiles += static_cast<int64_t>(n_t) * g.Hkv;
+        if (n_t > 0) n_pairs += g.Hkv;
     }
     out->units.clear();
     out->cta_off.clear();
@@ -492,88 +609,55 @@ void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geome
     for (int32_t s = 0; s < g.n_seq; ++s) max_cols = std::max(max_cols, (cu_q[s + 1] - cu_q[s]) * g.G);
     out->max_cols = max_cols;
     if (pairs.empty()) return;
+    const int32_t cap = std::max<int32_t>(max_ctas, 1);
+    int32_t n_sk = cap;
     // When every (sequence, kv head) pair has the same number of key tiles,
     // a grid of n CTAs splits no pair if n divides the pair count, and splits
     // every pair into equal chunks if the pair count divides n (and n / pairs
     // divides a pair's tiles).  A split pair costs its chunks a partial write
     // and its last chunk a merge (2-9% of such batches, measured), so with
-    // fit_grid the largest such grid down to 4/5 of max_ctas is taken.
-    if (fit_grid && max_ctas > 1) {
+    // fit_grid the largest such grid down to 4/5 of the cap is taken.
+    if (fit_grid && cap > 1) {
         int32_t tp = -1;
-        int64_t n_pairs = 0;
         bool uniform = true;
-        for (const Pair& pr : pairs) {
+        for (const DecPair& pr : pairs) {
             if (pr.n_t == 0) continue;
             if (tp < 0) tp = pr.n_t;
             uniform = uniform && pr.n_t == tp;
-            ++n_pairs;
         }
         if (uniform && n_pairs > 0) {
-            const int32_t lo = (max_ctas * 4 + 4) / 5;
-            for (int32_t n = max_ctas; n >= lo; --n) {
+            const int32_t lo = (cap * 4 + 4) / 5;
+            for (int32_t n = cap; n >= lo; --n) {
                 const bool whole = n_pairs % n == 0;
                 const bool equal = n % n_pairs == 0 && tp % (n / n_pairs) == 0;
                 if (whole || equal) {
-                    max_ctas = n;
+                    n_sk = n;
                     break;
                 }
             }
         }
     }
-    const int32_t n_cta = static_cast<int32_t>(std::max<int64_t>(
-        1, std::min<int64_t>(std::max<int32_t>(max_ctas, 1), std::max<int64_t>(total_tiles, 1))));
-    auto bound = [&](int64_t c) { return c * total_tiles / n_cta; };  // first tile of CTA c's stretch
-    auto make = [&](const Pair& pr, int32_t t0, int32_t n) {
-        DecUnit u;
-        u.q_tok0 = cu_q[pr.s];
-        u.nq = cu_q[pr.s + 1] - cu_q[pr.s];
-        u.k_row0 = cu_k[pr.s];
-        u.Lk = cu_k[pr.s + 1] - cu_k[pr.s];
-        u.kvh = pr.h;
-        u.tile0 = t0;
-        u.n_tiles = n;
-        u.part = -1;
-        u.group = -1;
-        u.chunk = 0;
-        u.n_chunks = 1;
-        u.seq = pr.s;
-        return u;
-    };
-    std::vector<std::vector<DecUnit>> per_cta(static_cast<size_t>(n_cta));
-    int64_t pos = 0;  // global index of the pair's first tile
+    n_sk = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(n_sk, std::max<int64_t>(total_tiles, 1))));
+    std::vector<std::vector<DecUnit>> per_cta(static_cast<size_t>(n_sk));
+    DecodeSchedule sk = *out;
+    if (total_tiles > 0) stream_k_cut(pairs, total_tiles, n_sk, cu_q, cu_k, &sk, &per_cta);
+    if (fit_grid && n_pairs > 0 && n_pairs <= cap) {
+        std::vector<std::vector<DecUnit>> pa_cta;
+        DecodeSchedule pa = *out;
+        pair_aligned_cut(pairs, cap, cu_q, cu_k, &pa, &pa_cta);
+        if (decode_schedule_cost(pa_cta, total_tiles) <= decode_schedule_cost(per_cta, total_tiles)) {
+            per_cta.swap(pa_cta);
+            sk = pa;
+        }
+    }
+    out->n_groups = sk.n_groups;
+    out->n_parts = sk.n_parts;
+    const int32_t n_cta = static_cast<int32_t>(per_cta.size());
     int32_t zero_rr = 0;
-    for (const Pair& pr : pairs) {
-        if (pr.n_t == 0) {
-            per_cta[static_cast<size_t>(zero_rr)].push_back(make(pr, 0, 0));
-            zero_rr = (zero_rr + 1) % n_cta;
-            continue;
-        }
-        // CTAs whose stretch meets [pos, pos + n_t)
-        int64_t c = std::min<int64_t>(n_cta - 1, pos * n_cta / total_tiles);
-        while (c > 0 && bound(c) > pos) --c;
-        while (c + 1 < n_cta && bound(c + 1) <= pos) ++c;
-        std::vector<std::pair<int64_t, DecUnit>> pieces;
-        int64_t t = pos;
-        const int64_t end = pos + pr.n_t;
-        while (t < end) {
-            const int64_t stop = std::min<int64_t>(end, bound(c + 1));
-            if (stop > t) pieces.push_back({c, make(pr, static_cast<int32_t>(t - pos), static_cast<int32_t>(stop - t))});
-            t = stop;
-            ++c;
-        }
-        const int32_t n_chunks = static_cast<int32_t>(pieces.size());
-        const int32_t group = n_chunks > 1 ? out->n_groups++ : -1;
-        const int32_t part0 = n_chunks > 1 ? out->n_parts : -1;
-        if (n_chunks > 1) out->n_parts += n_chunks;
-        for (int32_t i = 0; i < n_chunks; ++i) {
-            DecUnit& u = pieces[static_cast<size_t>(i)].second;
-            u.chunk = i;
-            u.n_chunks = n_chunks;
-            u.group = group;
-            u.part = n_chunks > 1 ? part0 + i : -1;
-            per_cta[static_cast<size_t>(pieces[static_cast<size_t>(i)].first)].push_back(u);
-        }
-        pos = end;
+    for (const DecPair& pr : pairs) {
+        if (pr.n_t != 0) continue;
+        add_pair_units(pr, {{zero_rr, 0, 0}}, cu_q, cu_k, out, &per_cta);
+        zero_rr = (zero_rr + 1) % n_cta;
     }
     out->cta_off.assign(static_cast<size_t>(n_cta) + 1, 0);
     for (int32_t c = 0; c < n_cta; ++c) {
@@ -1025,10 +1109,13 @@ opattn_status opattn_plan_run_paged(const opattn_plan* plan, const void* q, cons
     return launch_decode(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
 }
 
-opattn_status opattn_decode_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
-                                     int32_t Hq, int32_t Hkv, int32_t d, int32_t n_ctas, int32_t* units,
-                                     int64_t unit_capacity, int32_t* cta_offsets, int64_t* n_units_out,
-                                     int32_t* n_ctas_used) {
+}  // extern "C"
+
+namespace {
+opattn_status decode_schedule_out(const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
+                                  int32_t Hq, int32_t Hkv, int32_t d, int32_t n_ctas, bool fit_grid, int32_t* units,
+                                  int64_t unit_capacity, int32_t* cta_offsets, int64_t* n_units_out,
+                                  int32_t* n_ctas_used) {
     if (n_ctas <= 0 || !n_units_out || !n_ctas_used) return OPATTN_ERR_INVALID_ARG;
     Geometry g;
     opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
@@ -1036,7 +1123,7 @@ opattn_status opattn_decode_schedule(const int32_t* cu_seqlens_q, const int32_t*
     st = check_decode_geometry(cu_seqlens_q, g);
     if (st != OPATTN_OK) return st;
     DecodeSchedule sch;
-    build_decode_schedule(cu_seqlens_q, cu_seqlens_k, g, n_ctas, &sch);
+    build_decode_schedule(cu_seqlens_q, cu_seqlens_k, g, n_ctas, &sch, fit_grid);
     *n_units_out = static_cast<int64_t>(sch.units.size());
     *n_ctas_used = sch.n_cta;
     if (static_cast<int64_t>(sch.units.size()) > unit_capacity) return OPATTN_ERR_CAPACITY;
@@ -1046,6 +1133,25 @@ opattn_status opattn_decode_schedule(const int32_t* cu_seqlens_q, const int32_t*
         std::memcpy(cta_offsets, sch.cta_off.data(), sch.cta_off.size() * sizeof(int32_t));
     }
     return OPATTN_OK;
+}
+}  // namespace
+
+extern "C" {
+
+opattn_status opattn_decode_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
+                                     int32_t Hq, int32_t Hkv, int32_t d, int32_t n_ctas, int32_t* units,
+                                     int64_t unit_capacity, int32_t* cta_offsets, int64_t* n_units_out,
+                                     int32_t* n_ctas_used) {
+    return decode_schedule_out(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, n_ctas, false, units, unit_capacity,
+                               cta_offsets, n_units_out, n_ctas_used);
+}
+
+opattn_status opattn_decode_schedule_default(const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k,
+                                             int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, int32_t sms,
+                                             int32_t* units, int64_t unit_capacity, int32_t* cta_offsets,
+                                             int64_t* n_units_out, int32_t* n_ctas_used) {
+    return decode_schedule_out(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, sms, true, units, unit_capacity,
+                               cta_offsets, n_units_out, n_ctas_used);
 }
 
 }  // extern "C"

@@ -30,6 +30,7 @@ def test_header_declares_the_entry_points():
     for name in ["opattn_prefill", "opattn_prefill_checked", "opattn_prefill_noalloc", "opattn_plan_create",
                  "opattn_plan_run", "opattn_plan_destroy", "opattn_plan_info", "opattn_schedule",
                  "opattn_decode", "opattn_decode_checked", "opattn_decode_plan_create", "opattn_decode_schedule",
+                 "opattn_decode_schedule_default",
                  "opattn_decode_paged", "opattn_decode_paged_plan_create", "opattn_prefill_paged",
                  "opattn_prefill_paged_plan_create", "opattn_plan_run_paged", "opattn_version",
                  "opattn_status_string"]:

@@ -3,8 +3,10 @@
 Checked against brute-force enumeration: every (sequence, kv head, key tile)
 is covered by exactly one chunk, chunks of a pair are contiguous and
 numbered in tile order and sit on different CTAs, partial slots and merge
-groups are unique and dense, and every CTA streams the same number of key
-tiles to within one.
+groups are unique and dense, and (stream-K cut) every CTA streams the same
+number of key tiles to within one.  The default-grid schedule is checked for
+the same cover, for one chunk per CTA on small batches and for the fitted
+grid of a large uniform batch.
 """
 import ctypes
 
@@ -40,12 +42,9 @@ CASES = [
 ]
 
 
-@pytest.mark.parametrize("case", CASES)
-def test_chunks_cover_every_key_tile_once(case):
-    lq, lk, Hq, Hkv, n_cta = case
-    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
-    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
-    units, offs = pkg.opattn_decode_schedule(cu_q, cu_k, Hq, Hkv, 128, n_cta)
+def check_cover(lq, lk, Hkv, cu_q, cu_k, units, offs):
+    """Every (sequence, kv head, key tile) in exactly one chunk; chunks numbered in tile order, one per CTA;
+    partial slots contiguous per pair and dense; merge groups dense."""
     t = table(units)
     seen = {}
     for i in range(len(units)):
@@ -80,6 +79,17 @@ def test_chunks_cover_every_key_tile_once(case):
             parts += list(range(p0, p0 + n_chunks))
     assert sorted(groups) == list(range(len(groups)))
     assert sorted(parts) == list(range(len(parts)))
+    assert offs[-1] == len(units)
+    return t
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_chunks_cover_every_key_tile_once(case):
+    lq, lk, Hq, Hkv, n_cta = case
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_decode_schedule(cu_q, cu_k, Hq, Hkv, 128, n_cta)
+    t = check_cover(lq, lk, Hkv, cu_q, cu_k, units, offs)
     # every CTA streams floor or ceil of the mean number of key tiles
     total = int(t["n_tiles"].sum())
     n_used = len(offs) - 1
@@ -88,6 +98,49 @@ def test_chunks_cover_every_key_tile_once(case):
         assert n_used == min(n_cta, total)
         loads = np.array([t["n_tiles"][offs[c]:offs[c + 1]].sum() for c in range(n_used)])
         assert loads.min() >= total // n_used and loads.max() <= -(-total // n_used)
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_default_grid_schedule_covers_every_key_tile_once(case):
+    lq, lk, Hq, Hkv, sms = case
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_decode_schedule_default(cu_q, cu_k, Hq, Hkv, 128, sms)
+    check_cover(lq, lk, Hkv, cu_q, cu_k, units, offs)
+    assert 1 <= len(offs) - 1 <= sms
+
+
+def default_schedule(B, L, sms=152, Hq=64, Hkv=8):
+    cu_q = np.arange(B + 1, dtype=np.int32)
+    cu_k = (cu_q * L).astype(np.int32)
+    units, offs = pkg.opattn_decode_schedule_default(cu_q, cu_k, Hq, Hkv, 128, sms)
+    t = check_cover([1] * B, [L] * B, Hkv, cu_q, cu_k, units, offs)
+    return t, offs
+
+
+@pytest.mark.parametrize("B,L,ctas,chunks", [
+    (4, 1248, 128, {4}),     # 32 pairs of 10 tiles: 4 chunks of 2-3 tiles each, not 5-6 stream-K pieces
+    (12, 1500, 96, {1}),     # 96 pairs of 12 tiles: one CTA each, nothing split
+    (16, 2048, 128, {1}),    # 128 pairs of 16 tiles: one CTA each
+    (1, 6268, 136, {17}),    # 8 pairs of 49 tiles: 17 chunks of at most 3 tiles
+])
+def test_small_batches_get_one_chunk_per_cta(B, L, ctas, chunks):
+    """At most as many (sequence, kv head) pairs as SMs: the default grid cuts pair by pair, so no CTA
+    holds the end of one split pair and the start of the next (about 3.8 us more on GB300)."""
+    t, offs = default_schedule(B, L)
+    assert len(offs) - 1 == ctas
+    assert np.all(np.diff(offs) == 1)                       # one unit per CTA
+    assert set(int(c) for c in t["n_chunks"]) == chunks
+    n_t = -(-L // BN)
+    m = -(-n_t // max(chunks))
+    assert t["n_tiles"].max() == m and t["n_tiles"].min() >= n_t // max(chunks)
+
+
+def test_large_uniform_batch_keeps_the_fitted_stream_k_grid():
+    t, offs = default_schedule(64, 8192)                    # 512 pairs > 152 SMs
+    assert len(offs) - 1 == 128 and set(int(c) for c in t["n_chunks"]) == {1}
+    loads = np.array([t["n_tiles"][offs[c]:offs[c + 1]].sum() for c in range(128)])
+    assert loads.min() == loads.max() == 4 * 64
 
 
 def test_long_contexts_are_split_for_parallelism():
