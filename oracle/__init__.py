@@ -18,6 +18,9 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
+# A prebuilt variant of the library, loaded instead of building oracle.c: the
+# mutation tests point it at copies of oracle.c with a mistake planted in them.
+_OVERRIDE = os.environ.get("OPATTN_ORACLE_LIBRARY")
 _lock = threading.Lock()
 _lib = None
 
@@ -36,8 +39,11 @@ def _load():
     global _lib
     with _lock:
         if _lib is None:
-            build()
-            lib = ctypes.CDLL(_LIB)
+            if _OVERRIDE:
+                lib = ctypes.CDLL(_OVERRIDE)
+            else:
+                build()
+                lib = ctypes.CDLL(_LIB)
             p = ctypes.c_void_p
             i32, i64, f64 = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
             lib.oracle_attention_rows.argtypes = [p, p, p, p, p, i32, i32, i32, i32, f64,

@@ -32,7 +32,9 @@
  * Parity pins (test suite, CPU): length-1 rows, constant V, zero queries,
  * a hand-derived worked example, a dense masked-matrix formulation through
  * scipy on tiny inputs, chunk consistency, head-mapping and sequence
- * permutation invariants, and rows that see no key.
+ * permutation invariants, and rows that see no key.  A mutation test plants
+ * plausible mistakes in copies of this file and checks that a pin fails for
+ * each.
  */
 #include <math.h>
 #include <pthread.h>
