@@ -233,3 +233,34 @@ def test_paged_prefill_argument_errors(kwargs, status):
                                   args["seqlens_k"], 1, args["Hq"], args["Hkv"], args["d"], args["scale"],
                                   stream=0, check=False)
     assert st == status
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_default_grid_schedule_on_random_batches(seed):
+    """Seeded random ragged batches (empty sequences, Lq = 0, few and many pairs, 1 to 152 SMs): the
+    default-grid schedule covers every key tile exactly once, uses at most the SMs given, and when it
+    cuts pair by pair gives every CTA one chunk with keys."""
+    rng = np.random.default_rng(500 + seed)
+    G = int(rng.choice([1, 2, 4, 8, 16, 32]))
+    Hkv = int(rng.choice([1, 2, 4, 8]))
+    n_seq = int(rng.integers(1, 40))
+    max_q = 32 // G
+    lq = [int(rng.integers(0, max_q + 1)) for _ in range(n_seq)]
+    lk = [int(rng.integers(0, 20000)) if rng.random() < 0.9 else 0 for _ in range(n_seq)]
+    sms = int(rng.choice([1, 7, 64, 100, 152]))
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_decode_schedule_default(cu_q, cu_k, G * Hkv, Hkv, 128, sms)
+    if len(units) == 0:
+        assert sum(lq) == 0
+        return
+    t = check_cover(lq, lk, Hkv, cu_q, cu_k, units, offs)
+    n_used = len(offs) - 1
+    assert 1 <= n_used <= sms
+    with_keys = np.array([int((t["n_tiles"][offs[c]:offs[c + 1]] > 0).sum()) for c in range(n_used)])
+    pairs = sum(Hkv for s in range(n_seq) if lq[s] > 0 and lk[s] > 0)
+    if 0 < pairs <= sms and with_keys.max() == 1:
+        # pair-aligned: chunks of one pair differ by at most one tile
+        for (s, h) in {(int(a), int(b)) for a, b in zip(t["seq"], t["kvh"])}:
+            sizes = t["n_tiles"][(t["seq"] == s) & (t["kvh"] == h)]
+            assert sizes.max() - sizes.min() <= 1
