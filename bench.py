@@ -337,7 +337,11 @@ def run_ours(args, w):
     # back, all inside the timed region.  Two device buffer sets and separate
     # copy streams let step i + 1's input copy and step i - 1's output copy run
     # while step i computes, as a serving loop that stages the next batch would.
-    e2e_steps = max(3, min(args.steps, args.e2e_steps))
+    # As many steps as the device-timed region (unless --e2e-steps asks for
+    # fewer), so that the pipeline's fill (the first step's input copy) and
+    # drain (the last step's output copy) weigh as little as they do in a
+    # serving loop.
+    e2e_steps = max(3, min(args.steps, args.e2e_steps if args.e2e_steps > 0 else args.steps))
     hq = q.cpu().pin_memory()
     hk = k.cpu().pin_memory()
     hv = v.cpu().pin_memory()
@@ -487,7 +491,8 @@ def main(argv=None):
     ap.add_argument("--workload", default="llama3_70b",
                     help="tiny | llama3_8b | llama3_70b | bursty | chunked | decode_llama3_70b | "
                          "decode_llama3_8b | decode_spec4_llama3_70b | decode_llama3_70b_paged16")
-    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--e2e-steps", type=int, default=0,
+                    help="steps of the end-to-end measurement (default 0: as many as --steps)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--reference-step-seconds", type=float, default=3.0,
