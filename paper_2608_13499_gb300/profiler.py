@@ -549,7 +549,19 @@ def _colocation_section(reps: int) -> list:
         torch.cuda.empty_cache()
     lines += ["", f"Alone on all {sms} SMs: prefill {r['full_gpu_ms'][0]:.3f} ms, decode "
               f"{r['full_gpu_ms'][1]:.3f} ms per launch.", ""]
-    return lines
+    half = sms // 2
+    lines += [f"Other operator pairs, {half} + {sms - half} SMs (A + B):", "",
+              "| A | B | A ms: alone at budget / co-located (I) | B ms: alone at budget / co-located (I) | "
+              "speedup over time slicing |", "|---|---|---|---|---|"]
+    pairs = [(W.STANDARD["llama3_70b"](), False, W.STANDARD["llama3_8b"](), False),
+             (W.DECODE["decode_llama3_70b"](), True, W.DECODE["decode_llama3_8b"](), True)]
+    for w1, d1, w2, d2 in pairs:
+        r = colocate(w1, w2, half, sms - half, decode_a=d1, decode_b=d2, reps=reps)
+        lines.append(f"| {w1.name} | {w2.name} | {r['alone_ms'][0]:.3f} / {r['colocated_ms'][0]:.3f} "
+                     f"({r['interference'][0]:.3f}) | {r['alone_ms'][1]:.3f} / {r['colocated_ms'][1]:.3f} "
+                     f"({r['interference'][1]:.3f}) | {r['speedup']:.2f}x |")
+        torch.cuda.empty_cache()
+    return lines + [""]
 
 
 def main(argv=None):
