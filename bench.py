@@ -438,7 +438,8 @@ def run_ours(args, w):
             "flops_per_step": flops,
             "roofline": roofline,
             "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "steps": e2e_steps, "pipelined": "three buffer sets; copies overlap the neighbouring steps"},
+                    "steps": e2e_steps, "pipelined": "three buffer sets; copies overlap the neighbouring steps",
+                    "gpu_launches": 2 * e2e_steps},  # per one-shot call: the work-list upload and the attention kernel
             "cpu_baseline": cpu_base,
             "clocks": clocks,
             "gpu_launches": args.steps,
