@@ -185,6 +185,14 @@ def test_decode_plan_and_schedule_validate():
     st = lib.opattn_decode_schedule(cu.ctypes.data_as(ctypes.c_void_p), cu.ctypes.data_as(ctypes.c_void_p), 1,
                                     16, 2, 128, 0, None, 0, None, ctypes.byref(n_units), ctypes.byref(n_used))
     assert st == pkg.OPATTN_ERR_INVALID_ARG                             # n_ctas must be positive
+    st = lib.opattn_decode_schedule_default(cu.ctypes.data_as(ctypes.c_void_p), cu.ctypes.data_as(ctypes.c_void_p),
+                                            1, 16, 2, 128, 0, None, 0, None, ctypes.byref(n_units),
+                                            ctypes.byref(n_used))
+    assert st == pkg.OPATTN_ERR_INVALID_ARG                             # sms must be positive
+    st = lib.opattn_decode_schedule_default(cu.ctypes.data_as(ctypes.c_void_p), cu.ctypes.data_as(ctypes.c_void_p),
+                                            1, 16, 2, 64, 152, None, 0, None, ctypes.byref(n_units),
+                                            ctypes.byref(n_used))
+    assert st == pkg.OPATTN_ERR_UNSUPPORTED                             # the decode kernel is d = 128 only
     assert pkg.opattn_decode_checked(A, A, A, A, A, (0, 1), (0, 9), 1, 16, 2, 128, 0.1, stream=0,
                                      flags=0x40) == pkg.OPATTN_ERR_INVALID_ARG
 
