@@ -97,15 +97,25 @@ OPATTN_API opattn_status opattn_prefill(const void *q, const void *k, const void
  * allocate device memory: a serving engine that reserves almost all of HBM
  * for its KV cache and hands out memory only from its own pool, a process
  * whose device memory is capped by a quota, or a device without the
- * stream-ordered allocator.  Same arguments, computation and asynchrony as
+ * stream-ordered allocator.  Same arguments and computation as
  * opattn_prefill; the caller still provides q, k, v, o and lse.  The work
  * list and status word go to a fixed device array inside the library
  * (OPATTN_NOALLOC_MAX_UNITS work units of 32 bytes plus 8 KiB, about 1 MiB),
  * which every GPU that loads the library keeps until the process exits.  It
- * calls no cudaMalloc, cudaMallocAsync or cudaFree (the host side builds
- * the list in ordinary heap memory and copies it with cudaMemcpyAsync).
+ * calls no cudaMalloc, cudaMallocAsync or cudaFree, and no cudaHostAlloc
+ * either: the host side builds the list in ordinary heap memory and copies
+ * it with cudaMemcpyAsync.
+ *   - That copy from pageable memory may block the calling thread until the
+ *     runtime has staged the bytes (it can wait for work already queued on
+ *     `stream`); opattn_prefill, whose list sits in pinned memory, never
+ *     blocks.
+ *   - Not for stream capture: the copy reads heap memory that is freed when
+ *     the call returns, so a captured call could not be replayed.  A call on
+ *     a capturing stream returns OPATTN_ERR_INVALID_ARG before any device
+ *     work; use the opattn_plan_* calls for CUDA graphs.
  *   - The first call on a device looks up the array's device address with
- *     that device current; make that first call before any stream capture.
+ *     that device current and keeps it for later calls, so cudaDeviceReset
+ *     while the library is loaded is not supported.
  *   - All calls share the one array and each overwrites it: calls that
  *     overlap on the GPU (unordered streams, or several host threads) race,
  *     so order them on one stream or serialize them.
@@ -124,11 +134,14 @@ OPATTN_API opattn_status opattn_prefill_noalloc(const void *q, const void *k, co
  * Diagnostic variant: the same computation, then it synchronizes `stream`
  * and reads back the kernel's status word; returns OPATTN_ERR_TIMEOUT if a
  * bounded wait expired.  `flags` must be 0 except in the library's own
- * failure-path test, where OPATTN_FLAG_TEST_FORCE_TIMEOUT makes one kernel
- * wait run out on purpose (after ~20 ms) so that the error path is
- * exercised without hanging the GPU; outputs are then unspecified.
+ * failure-path tests, where OPATTN_FLAG_TEST_FORCE_TIMEOUT makes one wait of
+ * every CTA run out on purpose (after ~20 ms), and
+ * OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA only the one of CTA 0 (the other
+ * CTAs finish their work), so that the error path is exercised without
+ * hanging the GPU; outputs are then unspecified.
  */
 #define OPATTN_FLAG_TEST_FORCE_TIMEOUT 1u
+#define OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA 2u
 OPATTN_API opattn_status opattn_prefill_checked(const void *q, const void *k, const void *v, void *o, float *lse,
                                      const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
                                      int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
@@ -152,6 +165,16 @@ OPATTN_API opattn_status opattn_plan_create(opattn_plan **plan, const int32_t *c
 OPATTN_API opattn_status opattn_plan_run(const opattn_plan *plan, const void *q, const void *k, const void *v,
                               void *o, float *lse, float scale, void *stream);
 OPATTN_API opattn_status opattn_plan_destroy(opattn_plan *plan);
+/*
+ * Diagnostic run of a packed-K/V plan (prefill or decode): zeroes the plan's
+ * device status word, launches like opattn_plan_run with the test `flags` of
+ * opattn_prefill_checked, synchronizes `stream` and returns
+ * OPATTN_ERR_TIMEOUT if a bounded device wait expired.  Paged plans return
+ * OPATTN_ERR_INVALID_ARG.
+ */
+OPATTN_API opattn_status opattn_plan_run_checked(const opattn_plan *plan, const void *q, const void *k,
+                                                 const void *v, void *o, float *lse, float scale, void *stream,
+                                                 uint32_t flags);
 /* Number of work units and CTAs of a plan (either pointer may be NULL). */
 OPATTN_API opattn_status opattn_plan_info(const opattn_plan *plan, int64_t *n_units, int32_t *n_ctas);
 
@@ -213,11 +236,13 @@ OPATTN_API opattn_status opattn_decode_checked(const void *q, const void *k, con
  * plan is run, queried and destroyed with opattn_plan_run / _info / _destroy.
  * The plan owns the chunk partials, so two runs of one plan must not overlap
  * (run them on one stream).  A run is one kernel launch and nothing else: the
- * plan's merge counters are zeroed when it is created and every completed run
- * leaves them at zero, so runs can also be captured in a CUDA graph and
- * replayed.  Plan runs do not read the device status word; a run that hit a
- * device wait timeout leaves the counters undefined, and the plan must then
- * be destroyed rather than run again.
+ * plan's merge counters are zeroed when it is created and tagged with a
+ * launch epoch that the kernel itself advances when the launch's last CTA
+ * exits, so runs can also be captured in a CUDA graph and replayed.  A run
+ * that stopped early (a device wait timed out) leaves counts under its own
+ * epoch only, which later runs of the plan ignore: the plan stays usable.
+ * Plan runs do not read the device status word; opattn_plan_run_checked
+ * does.
  */
 OPATTN_API opattn_status opattn_decode_plan_create(opattn_plan **plan, const int32_t *cu_seqlens_q,
                                                    const int32_t *cu_seqlens_k, int32_t n_seq, int32_t Hq,

@@ -24,6 +24,7 @@ OPATTN_ERR_CUDA = 4
 OPATTN_ERR_TIMEOUT = 5
 OPATTN_ERR_CAPACITY = 6
 OPATTN_FLAG_TEST_FORCE_TIMEOUT = 1
+OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA = 2
 OPATTN_NOALLOC_MAX_UNITS = 32768
 
 UNIT_FIELDS = ("q_tok0", "n_tok", "k_row0", "Lk", "qlim0", "kvh", "n_tiles", "seq")
@@ -66,6 +67,8 @@ def load():
             lib.opattn_plan_create.argtypes = [ctypes.POINTER(P), P, P, i32, i32, i32, i32, i32]
             lib.opattn_plan_run.restype = ctypes.c_int
             lib.opattn_plan_run.argtypes = [P, P, P, P, P, P, f32, P]
+            lib.opattn_plan_run_checked.restype = ctypes.c_int
+            lib.opattn_plan_run_checked.argtypes = [P, P, P, P, P, P, f32, P, u32]
             lib.opattn_plan_destroy.restype = ctypes.c_int
             lib.opattn_plan_destroy.argtypes = [P]
             lib.opattn_plan_info.restype = ctypes.c_int
@@ -295,6 +298,11 @@ class Plan:
                                     _stream_handle(stream))
         if st != OPATTN_OK:
             raise OpattnError(st, "opattn_plan_run")
+
+    def run_checked(self, q, k, v, o, lse, scale: float, stream=None, flags: int = 0) -> int:
+        """C ``opattn_plan_run_checked`` (synchronous; returns the status code)."""
+        return int(load().opattn_plan_run_checked(self._h, _dptr(q), _dptr(k), _dptr(v), _dptr(o), _dptr(lse),
+                                                  float(scale), _stream_handle(stream), int(flags)))
 
     def run_paged(self, q, k_cache, v_cache, block_table, num_blocks: int, o, lse, scale: float, stream=None) -> None:
         st = load().opattn_plan_run_paged(self._h, _dptr(q), _dptr(k_cache), _dptr(v_cache), _dptr(block_table),

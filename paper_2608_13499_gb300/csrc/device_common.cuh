@@ -44,7 +44,41 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64
     }
 }
 
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+// Launch epoch of a work area (RunWords), read by one thread when the CTA
+// starts.  The launch's CTAs all read the same value: it only advances once
+// every one of them has passed run_exit.
+__device__ __forceinline__ uint32_t run_epoch(const RunWords* run) {
+    return *reinterpret_cast<const volatile uint32_t*>(&run->epoch);
+}
+
+// Called by one thread of every CTA after the CTA's last access to the work
+// area's counters: the last CTA of the launch to get here advances the
+// epoch for the next launch of the same work list.
+__device__ __forceinline__ void run_exit(RunWords* run, uint32_t epoch) {
+    __threadfence();
+    if (atomicAdd(&run->exits, 1u) == gridDim.x - 1u) {
+        run->exits = 0u;
+        __threadfence();
+        *reinterpret_cast<volatile uint32_t*>(&run->epoch) = epoch + 1u;
+    }
+}
+
+// Counts one arrival on a merge counter during launch epoch `epoch` and
+// returns the count including it.  The counter holds (epoch << 32 | count);
+// a value left by another epoch counts as zero.  The loop only retries while
+// another chunk of the same group updates the counter.
+__device__ __forceinline__ uint32_t count_arrival(unsigned long long* ctr, uint32_t epoch) {
+    unsigned long long old = *reinterpret_cast<volatile unsigned long long*>(ctr);
+    for (;;) {
+        const uint32_t have = static_cast<uint32_t>(old >> 32) == epoch ? static_cast<uint32_t>(old) : 0u;
+        const unsigned long long want = (static_cast<unsigned long long>(epoch) << 32) | (have + 1u);
+        const unsigned long long prev = atomicCAS(ctr, old, want);
+        if (prev == old) return have + 1u;
+        old = prev;
+    }
+}
+
+using EncodeTiledFn =CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 // cuTensorMapEncodeTiled from the driver (looked up once), or nullptr.

@@ -7,8 +7,11 @@
 
 #include <algorithm>
 #include <array>
+#include <chrono>
 #include <cmath>
 #include <cstdint>
+#include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <functional>
 #include <mutex>
@@ -21,7 +24,7 @@
 namespace opattn {
 namespace {
 
-constexpr int32_t kVersion = 10000;  // 1.0.0
+constexpr int32_t kVersion = 10100;  // 1.1.0
 
 struct Geometry {
     int32_t n_seq, Hq, Hkv, d, G, TPB;
@@ -84,6 +87,14 @@ constexpr int64_t kL2GroupBytes = 48ll << 20;
 // Greedy list scheduling in the given order: each unit goes to the CTA with
 // the least cost so far (ties: lower CTA index); a CTA's units keep the
 // order.  Makespan within mean load + largest unit.
+//
+// The least-loaded CTA comes from a bucket queue: loads only grow, the least
+// load only grows, and every load lies within the largest unit cost C of the
+// least one, so C + 1 circular buckets indexed by load hold every CTA
+// without collisions.  Each bucket is a bitset of CTAs; its lowest set bit is
+// the lowest CTA index at that load, which is the order of (load, index)
+// pairs.  Batches whose buckets would take more than kMaxBucketWords words
+// use a heap of (load, index) pairs instead.
 template <class U, class CostFn>
 void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std::vector<U>* units,
                std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
@@ -93,18 +104,52 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
     *n_cta_out = 0;
     if (n == 0) return;
     const int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(std::max<int32_t>(max_ctas, 1), n));
-    using Slot = std::pair<int64_t, int32_t>;
-    std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> heap;
-    for (int32_t c = 0; c < n_cta; ++c) heap.push({0, c});
     std::vector<int32_t> owner(static_cast<size_t>(n));
     std::vector<int32_t> per_cta(static_cast<size_t>(n_cta), 0);
-    for (int64_t i = 0; i < n; ++i) {
-        Slot sl = heap.top();
-        heap.pop();
-        owner[static_cast<size_t>(i)] = sl.second;
-        ++per_cta[static_cast<size_t>(sl.second)];
-        sl.first += cost(ordered[static_cast<size_t>(i)]);
-        heap.push(sl);
+    int64_t max_cost = 1;
+    for (const U& u : ordered) max_cost = std::max<int64_t>(max_cost, cost(u));
+    const size_t words = (static_cast<size_t>(n_cta) + 63) / 64;
+    constexpr size_t kMaxBucketWords = size_t{1} << 20;
+    const size_t n_buckets = static_cast<size_t>(max_cost) + 1;
+    if (n_buckets * words <= kMaxBucketWords) {
+        std::vector<uint64_t> bits(n_buckets * words, 0);
+        std::vector<int32_t> count(n_buckets, 0);
+        std::vector<int64_t> load(static_cast<size_t>(n_cta), 0);
+        for (int32_t c = 0; c < n_cta; ++c) bits[static_cast<size_t>(c) >> 6] |= uint64_t{1} << (c & 63);
+        count[0] = n_cta;
+        int64_t least = 0;  // least load of any CTA
+        size_t b = 0;       // its bucket, least mod n_buckets
+        for (int64_t i = 0; i < n; ++i) {
+            while (count[b] == 0) {
+                ++least;
+                if (++b == n_buckets) b = 0;
+            }
+            uint64_t* row = bits.data() + b * words;
+            size_t wi = 0;
+            while (row[wi] == 0) ++wi;
+            const int32_t c = static_cast<int32_t>(wi * 64 + static_cast<size_t>(__builtin_ctzll(row[wi])));
+            row[wi] &= row[wi] - 1;
+            --count[b];
+            owner[static_cast<size_t>(i)] = c;
+            ++per_cta[static_cast<size_t>(c)];
+            const int64_t nl = load[static_cast<size_t>(c)] + cost(ordered[static_cast<size_t>(i)]);
+            load[static_cast<size_t>(c)] = nl;
+            const size_t nb = static_cast<size_t>(nl % static_cast<int64_t>(n_buckets));
+            bits[nb * words + (static_cast<size_t>(c) >> 6)] |= uint64_t{1} << (c & 63);
+            ++count[nb];
+        }
+    } else {
+        using Slot = std::pair<int64_t, int32_t>;
+        std::priority_queue<Slot, std::vector<Slot>, std::greater<Slot>> heap;
+        for (int32_t c = 0; c < n_cta; ++c) heap.push({0, c});
+        for (int64_t i = 0; i < n; ++i) {
+            Slot sl = heap.top();
+            heap.pop();
+            owner[static_cast<size_t>(i)] = sl.second;
+            ++per_cta[static_cast<size_t>(sl.second)];
+            sl.first += cost(ordered[static_cast<size_t>(i)]);
+            heap.push(sl);
+        }
     }
     cta_off->assign(static_cast<size_t>(n_cta) + 1, 0);
     for (int32_t c = 0; c < n_cta; ++c)
@@ -126,58 +171,74 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
 // within a group, each to the CTA with the least cost so far.  A CTA runs its
 // units in that order, so at any time the CTAs work on one group and each
 // K/V tile comes from HBM about once; across the whole list the greedy
-// assignment keeps the makespan within mean load + largest unit.
+// assignment keeps the makespan within mean load + largest unit.  The
+// longest-first order within a group is a stable counting sort on the tile
+// count (O(units + tiles) per group).
 void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out) {
     const int32_t tpu = 2 * g.TPB;
-    std::vector<UnitRec> all;
-    std::vector<int32_t> group_of;  // per unit
-    int32_t max_cost = 0;
-    int32_t group = 0;
+    int64_t n_units = 0;
+    for (int32_t s = 0; s < g.n_seq; ++s) n_units += (static_cast<int64_t>(cu_q[s + 1] - cu_q[s]) + tpu - 1) / tpu;
+    n_units *= g.Hkv;
+    std::vector<UnitRec> all(static_cast<size_t>(n_units));
+    std::vector<size_t> group_start;  // index in `all` of each group's first unit
+    std::vector<int32_t> group_max;   // most key tiles of a unit in the group
     int64_t group_bytes = 0;
     const int64_t pair_row_bytes = 2 * static_cast<int64_t>(g.d) * 2;  // K and V, bf16
+    size_t n = 0;
     for (int32_t s = 0; s < g.n_seq; ++s) {
         const int32_t Lq = cu_q[s + 1] - cu_q[s];
         const int32_t Lk = cu_k[s + 1] - cu_k[s];
         const int32_t delta = Lk - Lq;
         if (Lq == 0) continue;
+        // the units of kv head 0; the other heads' differ only in the head
+        const size_t first = n;
+        int32_t seq_max = 0;
+        for (int32_t t0 = 0; t0 < Lq; t0 += tpu) {
+            const int32_t n_tok = std::min(tpu, Lq - t0);
+            const int32_t qlim0 = t0 + delta;
+            const int32_t last_key = std::min(qlim0 + n_tok - 1, Lk - 1);
+            const int32_t n_tiles = last_key < 0 ? 0 : last_key / kBlockN + 1;
+            seq_max = std::max(seq_max, n_tiles);
+            UnitRec& u = all[n++];
+            u.q_tok0 = cu_q[s] + t0;
+            u.n_tok = n_tok;
+            u.k_row0 = cu_k[s];
+            u.Lk = Lk;
+            u.qlim0 = qlim0;
+            u.kvh = 0;
+            u.n_tiles = n_tiles;
+            u.seq = s;
+        }
+        const size_t per_head = n - first;
+        const int64_t pair_bytes = static_cast<int64_t>(Lk) * pair_row_bytes;
         for (int32_t h = 0; h < g.Hkv; ++h) {
-            const int64_t pair_bytes = static_cast<int64_t>(Lk) * pair_row_bytes;
-            if (group_bytes > 0 && group_bytes + pair_bytes > kL2GroupBytes) {
-                ++group;
+            if (group_start.empty() || (group_bytes > 0 && group_bytes + pair_bytes > kL2GroupBytes)) {
+                group_start.push_back(first + static_cast<size_t>(h) * per_head);
+                group_max.push_back(0);
                 group_bytes = 0;
             }
             group_bytes += pair_bytes;
-            for (int32_t t0 = 0; t0 < Lq; t0 += tpu) {
-                const int32_t n_tok = std::min(tpu, Lq - t0);
-                const int32_t qlim0 = t0 + delta;
-                const int32_t last_key = std::min(qlim0 + n_tok - 1, Lk - 1);
-                const int32_t n_tiles = last_key < 0 ? 0 : last_key / kBlockN + 1;
-                max_cost = std::max(max_cost, n_tiles + 1);
-                UnitRec u;
-                u.q_tok0 = cu_q[s] + t0;
-                u.n_tok = n_tok;
-                u.k_row0 = cu_k[s];
-                u.Lk = Lk;
-                u.qlim0 = qlim0;
-                u.kvh = h;
-                u.n_tiles = n_tiles;
-                u.seq = s;
-                all.push_back(u);
-                group_of.push_back(group);
-            }
+            group_max.back() = std::max(group_max.back(), seq_max);
+            if (h == 0) continue;
+            UnitRec* dst = all.data() + first + static_cast<size_t>(h) * per_head;
+            std::memcpy(dst, all.data() + first, per_head * sizeof(UnitRec));
+            for (size_t i = 0; i < per_head; ++i) dst[i].kvh = h;
         }
+        n = first + static_cast<size_t>(g.Hkv) * per_head;
     }
-    // group by group, longest first within a group (stable)
-    std::vector<int64_t> idx(all.size());
-    for (size_t i = 0; i < idx.size(); ++i) idx[i] = static_cast<int64_t>(i);
-    std::stable_sort(idx.begin(), idx.end(), [&](int64_t a, int64_t b) {
-        if (group_of[static_cast<size_t>(a)] != group_of[static_cast<size_t>(b)])
-            return group_of[static_cast<size_t>(a)] < group_of[static_cast<size_t>(b)];
-        return all[static_cast<size_t>(a)].n_tiles > all[static_cast<size_t>(b)].n_tiles;
-    });
-    std::vector<UnitRec> ordered;
-    ordered.reserve(all.size());
-    for (int64_t i : idx) ordered.push_back(all[static_cast<size_t>(i)]);
+    // group by group, longest first within a group (stable counting sort)
+    std::vector<UnitRec> ordered(all.size());
+    std::vector<size_t> slot;
+    group_start.push_back(all.size());
+    for (size_t gi = 0; gi + 1 < group_start.size(); ++gi) {
+        const size_t b = group_start[gi], e = group_start[gi + 1];
+        const int32_t mx = group_max[gi];
+        slot.assign(static_cast<size_t>(mx) + 2, 0);
+        for (size_t i = b; i < e; ++i) ++slot[static_cast<size_t>(mx - all[i].n_tiles) + 1];  // rank 0 = most tiles
+        slot[0] = b;
+        for (size_t r = 1; r < slot.size(); ++r) slot[r] += slot[r - 1];
+        for (size_t i = b; i < e; ++i) ordered[slot[static_cast<size_t>(mx - all[i].n_tiles)]++] = all[i];
+    }
     list_pack(ordered, max_ctas, [](const UnitRec& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
               &out->n_cta);
 }
@@ -200,6 +261,49 @@ void pack_upload(const Schedule& s, const WorkLayout& w, uint8_t* dst) {
     std::memcpy(dst, s.cta_off.data(), s.cta_off.size() * sizeof(int32_t));
     std::memcpy(dst + w.off_units, s.units.data(), s.units.size() * sizeof(UnitRec));
 }
+
+// ------------------------------------------------------ OPATTN_LOG=1
+// With OPATTN_LOG set to anything but "0" in the environment, every schedule
+// the library builds prints one line on stderr: work units, CTAs, the largest
+// and mean CTA load and the largest unit (in the scheduler's cost, key tiles
+// + 1 per unit for prefill, key tiles for decode), and the host time from the
+// call's entry to the finished list.
+bool log_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("OPATTN_LOG");
+        return e != nullptr && e[0] != '\0' && !(e[0] == '0' && e[1] == '\0');
+    }();
+    return on;
+}
+using Clock = std::chrono::steady_clock;
+double us_since(Clock::time_point t0) {
+    return std::chrono::duration<double, std::micro>(Clock::now() - t0).count();
+}
+template <class U, class CostFn>
+void log_schedule(const char* what, const std::vector<U>& units, const std::vector<int32_t>& cta_off, CostFn cost,
+                  double host_us, const char* extra = "") {
+    if (!log_enabled()) return;
+    const size_t n_cta = cta_off.empty() ? 0 : cta_off.size() - 1;
+    int64_t total = 0, max_load = 0, max_unit = 0;
+    for (size_t c = 0; c < n_cta; ++c) {
+        int64_t load = 0;
+        for (int32_t i = cta_off[c]; i < cta_off[c + 1]; ++i) {
+            const int64_t u = cost(units[static_cast<size_t>(i)]);
+            load += u;
+            max_unit = std::max(max_unit, u);
+        }
+        total += load;
+        max_load = std::max(max_load, load);
+    }
+    std::fprintf(stderr,
+                 "opattn: %s: %zu units on %zu CTAs; CTA load max %lld mean %.1f (max/mean %.3f); largest unit %lld;"
+                 "%s host %.1f us\n",
+                 what, units.size(), n_cta, static_cast<long long>(max_load),
+                 n_cta ? static_cast<double>(total) / static_cast<double>(n_cta) : 0.0,
+                 total > 0 ? static_cast<double>(max_load) * static_cast<double>(n_cta) / static_cast<double>(total) : 0.0,
+                 static_cast<long long>(max_unit), extra, host_us);
+}
+int64_t prefill_cost(const UnitRec& u) { return u.n_tiles + 1; }
 
 // ---------------------------------------------------- pinned staging pool
 // The work list is built in mapped pinned memory and read from there by the
@@ -342,6 +446,7 @@ struct PagedArgs {
 opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
                            const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
                            cudaStream_t stream, uint32_t flags, bool checked, const PagedArgs* paged = nullptr) {
+    const Clock::time_point t_entry = Clock::now();
     Geometry g;
     opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
     if (st != OPATTN_OK) return st;
@@ -361,6 +466,7 @@ opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o,
 
     Schedule sch;
     build_schedule(cu_q, cu_k, g, sms, &sch);
+    log_schedule("prefill", sch.units, sch.cta_off, prefill_cost, us_since(t_entry));
     const WorkLayout w = work_layout(sch);
     Staging* stg = staging_acquire(w.upload_bytes);
     if (!stg) return OPATTN_ERR_CUDA;
@@ -412,6 +518,7 @@ int64_t count_units(const int32_t* cu_q, const Geometry& g) {
 opattn_status prefill_noalloc_impl(const void* q, const void* k, const void* v, void* o, float* lse,
                                    const int32_t* cu_q, const int32_t* cu_k, int32_t n_seq, int32_t Hq,
                                    int32_t Hkv, int32_t d, float scale, cudaStream_t stream) {
+    const Clock::time_point t_entry = Clock::now();
     Geometry g;
     opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
     if (st != OPATTN_OK) return st;
@@ -419,11 +526,21 @@ opattn_status prefill_noalloc_impl(const void* q, const void* k, const void* v, 
     st = check_tensors(q, k, v, o, lse, scale, g);
     if (st != OPATTN_OK) return st;
     if (count_units(cu_q, g) > kNoAllocMaxUnits) return OPATTN_ERR_CAPACITY;
+    // The list is copied from heap memory freed on return, which a captured
+    // graph could not replay.
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const cudaError_t ce = cudaStreamIsCapturing(stream, &cs);
+    if (ce != cudaSuccess) {
+        (void)cudaGetLastError();
+        return ce == cudaErrorStreamCaptureImplicit ? OPATTN_ERR_INVALID_ARG : OPATTN_ERR_CUDA;
+    }
+    if (cs != cudaStreamCaptureStatusNone) return OPATTN_ERR_INVALID_ARG;
     const int sms = device_sm_count();
     if (sms <= 0) return OPATTN_ERR_CUDA;
 
     Schedule sch;
     build_schedule(cu_q, cu_k, g, std::min(sms, kNoAllocMaxCtas), &sch);
+    log_schedule("prefill (no-alloc)", sch.units, sch.cta_off, prefill_cost, us_since(t_entry));
     const WorkLayout w = work_layout(sch);
     void* scratch = nullptr;
     size_t scratch_bytes = 0;
@@ -670,20 +787,22 @@ void build_decode_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geome
 }
 
 // Device work area: [cta_off | pad 32 | units | counters (2 per group: one per
-// softmax warpgroup) | status |
-// pad 256 | part_lse (n_parts x kDecCols) | part_o (n_parts x kDecCols x d)].
-// The counters and the status word are contiguous.  One-shot calls zero them
-// with the work-list upload before every launch; a plan zeroes them once when
-// it is created, and every launch that completes leaves the counters at zero
-// (the merging chunk resets its counter), so plan runs need no memset.
+// softmax warpgroup, 8 bytes each) | run words (epoch, exits) | status | pad 256 |
+// part_lse (n_parts x kDecCols) | part_o (n_parts x kDecCols x d)].  The
+// counters, the run words and the status word are contiguous.  One-shot calls
+// zero them with the work-list upload; a plan zeroes them once when it is
+// created.  Counters are tagged with the launch epoch, which the kernel
+// advances itself (RunWords), so plan runs need no memset, and a run that
+// stopped early leaves no count that a later run would take for its own.
 struct DecodeLayout {
-    size_t off_units, off_counters, off_status, off_part_lse, off_part_o, bytes, upload_bytes, zero_bytes;
+    size_t off_units, off_counters, off_run, off_status, off_part_lse, off_part_o, bytes, upload_bytes, zero_bytes;
 };
 DecodeLayout decode_layout(const DecodeSchedule& s) {
     DecodeLayout w;
     w.off_units = (s.cta_off.size() * sizeof(int32_t) + 31) / 32 * 32;
-    w.off_counters = w.off_units + s.units.size() * sizeof(DecUnit);
-    w.off_status = w.off_counters + 2 * static_cast<size_t>(s.n_groups) * sizeof(int32_t);
+    w.off_counters = w.off_units + s.units.size() * sizeof(DecUnit);  // a multiple of 16
+    w.off_run = w.off_counters + 2 * static_cast<size_t>(s.n_groups) * sizeof(unsigned long long);
+    w.off_status = w.off_run + sizeof(RunWords);
     w.upload_bytes = w.off_counters;
     w.zero_bytes = w.off_status + sizeof(int32_t) - w.off_counters;
     w.off_part_lse = (w.off_status + sizeof(int32_t) + 255) / 256 * 256;
@@ -714,7 +833,8 @@ DecodeLaunchArgs make_decode_args(const void* q, const void* k, const void* v, v
     a.cta_off = reinterpret_cast<const int32_t*>(work);
     a.n_cta = n_cta;
     a.max_cols = max_cols;
-    a.counters = reinterpret_cast<int32_t*>(work + w.off_counters);
+    a.counters = reinterpret_cast<unsigned long long*>(work + w.off_counters);
+    a.run = reinterpret_cast<RunWords*>(work + w.off_run);
     a.part_lse = reinterpret_cast<float*>(work + w.off_part_lse);
     a.part_o = reinterpret_cast<float*>(work + w.off_part_o);
     a.status = reinterpret_cast<int32_t*>(work + w.off_status);
@@ -726,9 +846,18 @@ DecodeLaunchArgs make_decode_args(const void* q, const void* k, const void* v, v
     return a;
 }
 
+void log_decode_schedule(const char* what, const DecodeSchedule& s, double host_us) {
+    if (!log_enabled()) return;
+    char extra[96];
+    std::snprintf(extra, sizeof extra, " %d split pairs, %d partials;", s.n_groups, s.n_parts);
+    log_schedule(what, s.units, s.cta_off, [](const DecUnit& u) { return static_cast<int64_t>(u.n_tiles); }, host_us,
+                 extra);
+}
+
 opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
                           const int32_t* cu_k, int32_t n_seq, int32_t Hq, int32_t Hkv, int32_t d, float scale,
                           cudaStream_t stream, uint32_t flags, bool checked, const PagedArgs* paged = nullptr) {
+    const Clock::time_point t_entry = Clock::now();
     Geometry g;
     opattn_status st = check_geometry(cu_q, cu_k, n_seq, Hq, Hkv, d, &g);
     if (st != OPATTN_OK) return st;
@@ -750,6 +879,7 @@ opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, 
 
     DecodeSchedule sch;
     build_decode_schedule(cu_q, cu_k, g, sms, &sch, /*fit_grid=*/true);
+    log_decode_schedule("decode", sch, us_since(t_entry));
     const DecodeLayout w = decode_layout(sch);
     Staging* stg = staging_acquire(w.upload_bytes);
     if (!stg) return OPATTN_ERR_CUDA;
@@ -839,8 +969,10 @@ opattn_status opattn_prefill_checked(const void* q, const void* k, const void* v
                                      const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
                                      int32_t Hq, int32_t Hkv, int32_t d, float scale, void* stream,
                                      uint32_t flags) {
-    if (flags & ~OPATTN_FLAG_TEST_FORCE_TIMEOUT) return OPATTN_ERR_INVALID_ARG;
-    const uint32_t kflags = (flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u;
+    if (flags & ~(OPATTN_FLAG_TEST_FORCE_TIMEOUT | OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA))
+        return OPATTN_ERR_INVALID_ARG;
+    const uint32_t kflags = ((flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u) |
+                            ((flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA) ? kFlagForceTimeoutFirstCta : 0u);
     return prefill_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
                         static_cast<cudaStream_t>(stream), kflags, true);
 }
@@ -866,7 +998,9 @@ opattn_status opattn_plan_create(opattn_plan** plan, const int32_t* cu_seqlens_q
             return OPATTN_ERR_CUDA;
         }
         const int32_t cap = max_ctas > 0 ? std::min(max_ctas, sms) : sms;
+        const Clock::time_point t0 = Clock::now();
         build_schedule(cu_seqlens_q, cu_seqlens_k, g, cap, &p->sch);
+        log_schedule("prefill plan", p->sch.units, p->sch.cta_off, prefill_cost, us_since(t0));
         p->w = work_layout(p->sch);
         std::vector<uint8_t> host(p->w.bytes, 0);
         pack_upload(p->sch, p->w, host.data());
@@ -884,22 +1018,55 @@ opattn_status opattn_plan_create(opattn_plan** plan, const int32_t* cu_seqlens_q
     return OPATTN_OK;
 }
 
-opattn_status opattn_plan_run(const opattn_plan* plan, const void* q, const void* k, const void* v, void* o,
-                              float* lse, float scale, void* stream) {
-    if (!plan) return OPATTN_ERR_INVALID_ARG;
-    if (plan->g.total_q == 0) return OPATTN_OK;
+}  // extern "C"
+
+namespace {
+// Launch of a packed-K/V plan with kernel flags (0 for opattn_plan_run).
+opattn_status plan_launch(const opattn_plan* plan, const void* q, const void* k, const void* v, void* o, float* lse,
+                          float scale, cudaStream_t stream, uint32_t kflags) {
     opattn_status st = check_tensors(q, k, v, o, lse, scale, plan->g);
     if (st != OPATTN_OK) return st;
     if (plan->block_size > 0) return OPATTN_ERR_INVALID_ARG;  // paged plans run with opattn_plan_run_paged
     uint8_t* work = static_cast<uint8_t*>(plan->work);
-    const cudaStream_t st_ = static_cast<cudaStream_t>(stream);
     if (plan->decode) {
-        const DecodeLaunchArgs a =
-            make_decode_args(q, k, v, o, lse, plan->g, scale, work, plan->dw, plan->dsch.n_cta, plan->dsch.max_cols, 0u);
-        return launch_decode(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+        const DecodeLaunchArgs a = make_decode_args(q, k, v, o, lse, plan->g, scale, work, plan->dw, plan->dsch.n_cta,
+                                                    plan->dsch.max_cols, kflags);
+        return launch_decode(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
     }
-    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, work, plan->w, plan->sch.n_cta, 0u);
-    return launch_prefill(a, st_) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, work, plan->w, plan->sch.n_cta, kflags);
+    return launch_prefill(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
+}
+}  // namespace
+
+extern "C" {
+
+opattn_status opattn_plan_run(const opattn_plan* plan, const void* q, const void* k, const void* v, void* o,
+                              float* lse, float scale, void* stream) {
+    if (!plan) return OPATTN_ERR_INVALID_ARG;
+    if (plan->g.total_q == 0) return OPATTN_OK;
+    return plan_launch(plan, q, k, v, o, lse, scale, static_cast<cudaStream_t>(stream), 0u);
+}
+
+opattn_status opattn_plan_run_checked(const opattn_plan* plan, const void* q, const void* k, const void* v, void* o,
+                                      float* lse, float scale, void* stream, uint32_t flags) {
+    if (!plan) return OPATTN_ERR_INVALID_ARG;
+    if (flags & ~(OPATTN_FLAG_TEST_FORCE_TIMEOUT | OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA))
+        return OPATTN_ERR_INVALID_ARG;
+    if (plan->block_size > 0) return OPATTN_ERR_INVALID_ARG;
+    if (plan->g.total_q == 0) return OPATTN_OK;
+    const uint32_t kflags = ((flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u) |
+                            ((flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA) ? kFlagForceTimeoutFirstCta : 0u);
+    const cudaStream_t st_ = static_cast<cudaStream_t>(stream);
+    int32_t* status = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(plan->work) +
+                                                 (plan->decode ? plan->dw.off_status : plan->w.off_status));
+    if (cudaMemsetAsync(status, 0, sizeof(int32_t), st_) != cudaSuccess) return OPATTN_ERR_CUDA;
+    opattn_status st = plan_launch(plan, q, k, v, o, lse, scale, st_, kflags);
+    if (st != OPATTN_OK) return st;
+    int32_t dev_status = 0;
+    if (cudaMemcpyAsync(&dev_status, status, sizeof(int32_t), cudaMemcpyDeviceToHost, st_) != cudaSuccess ||
+        cudaStreamSynchronize(st_) != cudaSuccess)
+        return OPATTN_ERR_CUDA;
+    return dev_status == kDevOk ? OPATTN_OK : OPATTN_ERR_TIMEOUT;
 }
 
 opattn_status opattn_plan_destroy(opattn_plan* plan) {
@@ -932,7 +1099,9 @@ opattn_status opattn_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seq
     opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
     if (st != OPATTN_OK) return st;
     Schedule sch;
+    const Clock::time_point t0 = Clock::now();
     build_schedule(cu_seqlens_q, cu_seqlens_k, g, n_ctas, &sch);
+    log_schedule("prefill schedule", sch.units, sch.cta_off, prefill_cost, us_since(t0));
     *n_units_out = static_cast<int64_t>(sch.units.size());
     *n_ctas_used = sch.n_cta;
     if (static_cast<int64_t>(sch.units.size()) > unit_capacity) return OPATTN_ERR_CAPACITY;
@@ -954,8 +1123,10 @@ opattn_status opattn_decode(const void* q, const void* k, const void* v, void* o
 opattn_status opattn_decode_checked(const void* q, const void* k, const void* v, void* o, float* lse,
                                     const int32_t* cu_seqlens_q, const int32_t* cu_seqlens_k, int32_t n_seq,
                                     int32_t Hq, int32_t Hkv, int32_t d, float scale, void* stream, uint32_t flags) {
-    if (flags & ~OPATTN_FLAG_TEST_FORCE_TIMEOUT) return OPATTN_ERR_INVALID_ARG;
-    const uint32_t kflags = (flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u;
+    if (flags & ~(OPATTN_FLAG_TEST_FORCE_TIMEOUT | OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA))
+        return OPATTN_ERR_INVALID_ARG;
+    const uint32_t kflags = ((flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT) ? kFlagForceTimeout : 0u) |
+                            ((flags & OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA) ? kFlagForceTimeoutFirstCta : 0u);
     return decode_impl(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, scale,
                        static_cast<cudaStream_t>(stream), kflags, true);
 }
@@ -992,7 +1163,9 @@ opattn_status decode_plan_create(opattn_plan** plan, const int32_t* cu_q, const 
         const int32_t cap = max_ctas > 0 ? std::min(max_ctas, sms) : sms;
         // an explicit SM budget is kept exactly; the default grid may shrink
         // a little so that a uniform batch splits no pair
+        const Clock::time_point t0 = Clock::now();
         build_decode_schedule(cu_q, cu_k, g, cap, &p->dsch, /*fit_grid=*/max_ctas == 0);
+        log_decode_schedule("decode plan", p->dsch, us_since(t0));
         p->dw = decode_layout(p->dsch);
         // the work list, then the counters and the status word at zero
         const size_t init_bytes = p->dw.off_counters + p->dw.zero_bytes;

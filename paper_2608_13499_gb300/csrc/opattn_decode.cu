@@ -119,7 +119,8 @@ struct DParams {
     float* lse;
     int32_t Hq, G, g_shift;  // G = 1 << g_shift
     float scale_log2;         // softmax scale * log2(e)
-    int32_t* counters;
+    unsigned long long* counters;
+    RunWords* run;
     float* part_o;
     float* part_lse;
     int32_t* status;
@@ -233,7 +234,7 @@ __device__ __forceinline__ void dec_mma(const DParams& p, int ubeg, int uend, ui
     uint32_t sbuf = 0;  // S buffer of the next S MMA (tiles are scored in order)
     uint32_t q_uses[2] = {0u, 0u};
     bool ok = true;
-    if (p.flags & kFlagForceTimeout)
+    if ((p.flags & kFlagForceTimeout) || ((p.flags & kFlagForceTimeoutFirstCta) && blockIdx.x == 0))
         ok = __all_sync(0xFFFFFFFFu, bounded_wait(bar(C::kBarNever), 0u, abort_flag, p.status, kForcedLimitNs));
 
     for (int ui = ubeg; ui < uend && ok; ++ui) {
@@ -356,7 +357,7 @@ __device__ __forceinline__ int64_t out_row(const DParams& p, const DecUnit& u, i
 // warpgroup, which is also its TMEM lane and the key of the tile it scores.
 template <int NCOL>
 __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend, uint32_t tmem, uint32_t sP,
-                                            float* sRed, uint32_t sBar, int wg, int tid,
+                                            float* sRed, uint32_t sBar, int wg, int tid, uint32_t epoch,
                                             volatile int32_t* abort_flag) {
     using C = DCfg;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
@@ -572,14 +573,9 @@ __device__ __forceinline__ void dec_softmax(const DParams& p, int ubeg, int uend
         __threadfence();
         ptx::bar_sync(kBarWG, kWGThreads);
         bool last = false;
-        // Each warpgroup counts the chunks of its own columns.  The chunk that
-        // finishes last has seen every arrival of this launch on its counter
-        // and sets it back to zero for the next launch of the same work list.
-        if (tid == 0) {
-            int32_t* counter = p.counters + 2 * u.group + wg;
-            last = atomicAdd(counter, 1) == u.n_chunks - 1;
-            if (last) *counter = 0;
-        }
+        // Each warpgroup counts the chunks of its own columns; the chunk that
+        // brings its counter to n_chunks in this launch's epoch merges.
+        if (tid == 0) last = count_arrival(p.counters + 2 * u.group + wg, epoch) == static_cast<uint32_t>(u.n_chunks);
         last = ptx::bar_red_or(kBarWG, kWGThreads, last);
         if (!last) continue;
         // This unit finished last: merge the (sequence, kv head)'s partials,
@@ -671,6 +667,7 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
     float* sRed = reinterpret_cast<float*>(gbase + C::kRedOff);
     volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(gbase + C::kMiscOff);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(gbase + C::kMiscOff + 4);
+    volatile uint32_t* epoch_slot = reinterpret_cast<volatile uint32_t*>(gbase + C::kMiscOff + 8);
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
@@ -695,6 +692,7 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
         ptx::mbar_init(sBar + 8u * C::kBarDrain, 1);
         ptx::mbar_init(sBar + 8u * C::kBarNever, 1);
         *abort_flag = 0;
+        *epoch_slot = run_epoch(p.run);
         ptx::fence_mbar_init();
     }
     if (tid < static_cast<int>(2 * kWGThreads)) {
@@ -718,11 +716,12 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    const uint32_t epoch = *epoch_slot;
     const int ubeg = p.cta_off[blockIdx.x];
     const int uend = p.cta_off[blockIdx.x + 1];
 
     if (warp < 8) {
-        dec_softmax<NCOL>(p, ubeg, uend, tmem, sP, sRed, sBar, warp >> 2, tid & 127, abort_flag);
+        dec_softmax<NCOL>(p, ubeg, uend, tmem, sP, sRed, sBar, warp >> 2, tid & 127, epoch, abort_flag);
     } else if (warp == kWarpProducerDec) {
         dec_producer<false>(&tmQ, &tmK, p, ubeg, uend, sQ, sK, sBar, lane, abort_flag);
     } else if (warp == kWarpProducerVDec) {
@@ -737,6 +736,7 @@ __global__ void __launch_bounds__(kThreadsDec, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);
     }
+    if (tid == 0) run_exit(p.run, epoch);
 }
 
 template <int NCOL>
@@ -798,6 +798,7 @@ int launch_decode(const DecodeLaunchArgs& a, cudaStream_t stream) {
     kp.g_shift = g_shift;
     kp.scale_log2 = a.scale * kLog2eDec;
     kp.counters = a.counters;
+    kp.run = a.run;
     kp.part_o = a.part_o;
     kp.part_lse = a.part_lse;
     kp.status = a.status;

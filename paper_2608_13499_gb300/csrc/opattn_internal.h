@@ -35,9 +35,24 @@ static_assert(sizeof(UnitRec) == 32, "UnitRec must stay 32 bytes");
 constexpr int32_t kDevOk = 0;
 constexpr int32_t kDevTimeout = 1;
 
-// Test-only launch flag: the MMA warp waits on a barrier nothing arrives on,
-// so the bounded-wait path runs (short limit, error status, clean exit).
+// Test-only launch flags: the MMA warp waits on a barrier nothing arrives on,
+// so the bounded-wait path runs (short limit, error status, clean exit); in
+// every CTA, or only in CTA 0 (the other CTAs finish their units, which
+// leaves the merge counters of a split launch part-counted).
 constexpr uint32_t kFlagForceTimeout = 1u;
+constexpr uint32_t kFlagForceTimeoutFirstCta = 2u;
+
+// Run bookkeeping of a work area whose kernel counts chunk arrivals (the
+// split-KV merge): run[0] is the launch epoch, run[1] the CTAs of the current
+// launch that have exited.  Every CTA reads the epoch when it starts; the
+// last CTA to exit advances it.  A merge counter holds (epoch << 32 | count),
+// and a counter written under another epoch counts as zero, so a launch that
+// stopped early (a wait timed out) leaves nothing behind that a later launch
+// of the same work list could miscount.  Both words start at zero.
+struct RunWords {
+    uint32_t epoch;
+    uint32_t exits;
+};
 
 struct LaunchArgs {
     const void* q;
@@ -111,7 +126,8 @@ struct DecodeLaunchArgs {
     const int32_t* cta_off;   // device, n_cta + 1
     int32_t n_cta;
     int32_t max_cols;         // largest G * Lq of the batch (<= kDecCols)
-    int32_t* counters;        // device, two per split (sequence, kv head), zero at launch
+    unsigned long long* counters;  // device, two per split (sequence, kv head), zeroed once
+    RunWords* run;            // device, zeroed once
     float* part_o;            // device, [parts][kDecCols][kDecHeadDim]
     float* part_lse;          // device, [parts][kDecCols] (log2 domain)
     int32_t* status;          // device

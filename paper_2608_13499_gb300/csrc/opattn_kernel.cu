@@ -305,7 +305,7 @@ __device__ __forceinline__ void run_mma(const KParams& p, int ubeg, int uend, ui
         return __all_sync(0xFFFFFFFFu, bounded_wait(bar(b), parity, abort_flag, p.status, kWaitLimitNs));
     };
     bool ok = true;
-    if (p.flags & kFlagForceTimeout)
+    if ((p.flags & kFlagForceTimeout) || ((p.flags & kFlagForceTimeoutFirstCta) && blockIdx.x == 0))
         ok = __all_sync(0xFFFFFFFFu, bounded_wait(bar(C::kBarNever), 0u, abort_flag, p.status, kForcedLimitNs));
 
     for (int ui = ubeg; ui < uend && ok; ++ui) {

@@ -28,7 +28,7 @@ def declared_symbols():
 def test_header_declares_the_entry_points():
     syms = declared_symbols()
     for name in ["opattn_prefill", "opattn_prefill_checked", "opattn_prefill_noalloc", "opattn_plan_create",
-                 "opattn_plan_run", "opattn_plan_destroy", "opattn_plan_info", "opattn_schedule",
+                 "opattn_plan_run", "opattn_plan_run_checked", "opattn_plan_destroy", "opattn_plan_info", "opattn_schedule",
                  "opattn_decode", "opattn_decode_checked", "opattn_decode_plan_create", "opattn_decode_schedule",
                  "opattn_decode_schedule_default",
                  "opattn_decode_paged", "opattn_decode_paged_plan_create", "opattn_prefill_paged",
@@ -44,7 +44,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_version_and_status_strings(lib):
-    assert pkg.opattn_version() == 10000
+    assert pkg.opattn_version() == 10100
     assert pkg.status_string(0) == "ok"
     for code in range(1, 7):
         assert pkg.status_string(code) not in ("ok", "unknown status")

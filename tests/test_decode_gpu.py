@@ -156,8 +156,9 @@ def test_plan_repeat_runs_on_a_side_stream():
 
 
 def test_plan_run_replays_from_a_cuda_graph():
-    """A decode plan run is one kernel launch that leaves its merge counters at zero, so a
-    captured run replays correctly, over key ranges split into up to 19 chunks."""
+    """A decode plan run is one kernel launch that advances its own launch epoch (the merge
+    counters are tagged with it), so a captured run replays correctly, over key ranges split
+    into up to 19 chunks."""
     w = custom("dec_graph", [1, 1, 1], [6268, 512, 3000], 64, 8, seed=16)
     q, k, v = W.make_inputs(w, "cuda")
     o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
@@ -190,6 +191,30 @@ def test_forced_timeout_reports_and_context_survives():
     assert pkg.opattn_decode_checked(q, k, v, o, lse, w.cu_q, w.cu_k, 1, 16, 2, 128, w.scale) == pkg.OPATTN_OK
     o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
     check(o, lse, o_ref, lse_ref, "after timeout")
+
+
+def test_plan_stays_correct_after_a_run_that_stopped_early():
+    """CTA 0 of a plan run gives up on a wait (test flag, ~20 ms) while the other CTAs finish their
+    chunks, so the split pairs' merge counters are left part-counted.  The counters carry the launch
+    epoch, which the kernel advances, so the following runs of the same plan ignore those counts."""
+    w = custom("dec_partial_abort", [1, 1, 1], [6268, 512, 3000], 64, 8, seed=17)
+    q, k, v = W.make_inputs(w, "cuda")
+    o_ref, lse_ref = oracle.attention(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale)
+    with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=True) as plan:
+        units, offs = pkg.opattn_decode_schedule_default(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d,
+                                                         torch.cuda.get_device_properties(0).multi_processor_count)
+        assert len(units) == plan.n_units
+        first = units[offs[0]:offs[1]]
+        assert (first[:, pkg.DEC_UNIT_FIELDS.index("n_chunks")] > 1).any()  # CTA 0 holds a chunk of a split pair
+        o = torch.empty((w.total_q, w.Hq, w.d), dtype=torch.bfloat16, device="cuda")
+        lse = torch.empty((w.total_q, w.Hq), dtype=torch.float32, device="cuda")
+        st = plan.run_checked(q, k, v, o, lse, w.scale, flags=pkg.OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA)
+        assert st == pkg.OPATTN_ERR_TIMEOUT
+        for i in range(3):
+            o.fill_(float("nan"))
+            lse.fill_(float("nan"))
+            assert plan.run_checked(q, k, v, o, lse, w.scale) == pkg.OPATTN_OK
+            check(o, lse, o_ref, lse_ref, f"run {i} after the early stop")
 
 
 @pytest.mark.parametrize("name", sorted(W.DECODE))

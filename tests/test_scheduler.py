@@ -88,7 +88,24 @@ def expected_order(lq, lk, Hkv, d, G):
     return sorted(keys, key=lambda k: (k[0], -k[1]))
 
 
-@pytest.mark.parametrize("case", CASES + [(W.chunked().q_lens, W.chunked().k_lens, 32, 8, 128, 152)])
+def random_cases(n, seed=123):
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        Hkv = int(rng.choice([1, 2, 8]))
+        G = int(rng.choice([1, 3, 4, 8, 16]))
+        d = int(rng.choice([64, 128]))
+        n_seq = int(rng.integers(1, 12))
+        lq = [int(x) for x in rng.integers(0, 3000, n_seq)]
+        lk = [max(0, q + int(rng.integers(-50, 9000))) for q in lq]
+        out.append((lq, lk, G * Hkv, Hkv, d, int(rng.choice([1, 5, 64, 152, 1000]))))
+    return out
+
+
+# The last case's loads span more buckets than the bucket queue takes
+# (1024 CTAs x 70K-tile units), so the scheduler uses its heap there.
+@pytest.mark.parametrize("case", CASES + [(W.chunked().q_lens, W.chunked().k_lens, 32, 8, 128, 152)] +
+                         random_cases(24) + [([512000], [9000000], 1, 1, 64, 1024)])
 def test_group_major_list_assignment(case):
     lq, lk, Hq, Hkv, d, n_cta = case
     cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
@@ -156,3 +173,29 @@ def test_standard_workload_unit_counts():
     w = W.tiny()
     units, _ = pkg.opattn_schedule(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, 152)
     assert len(units) == 6
+
+
+def test_opattn_log_prints_work_list_statistics():
+    """OPATTN_LOG=1 makes every schedule print one line on stderr: units, CTAs, largest and
+    mean CTA load, largest unit, host time (checked on the host-only scheduler)."""
+    import re
+    import subprocess
+    import sys
+    code = ("import paper_2608_13499_gb300 as pkg\n"
+            "units, offs = pkg.opattn_schedule([0, 300, 700], [0, 300, 900], 32, 8, 128, 5)\n"
+            "cost = units[:, 6].astype(int) + 1\n"
+            "loads = [int(cost[offs[c]:offs[c + 1]].sum()) for c in range(len(offs) - 1)]\n"
+            "print(len(units), len(offs) - 1, max(loads), sum(loads), int(cost.max()))\n")
+    env = dict(__import__("os").environ, OPATTN_LOG="1")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, check=True)
+    n, n_cta, mx, total, biggest = map(int, r.stdout.split())
+    lines = [ln for ln in r.stderr.splitlines() if ln.startswith("opattn:")]
+    assert len(lines) == 2  # the binding asks for the size first, then for the list
+    m = re.match(r"opattn: prefill schedule: (\d+) units on (\d+) CTAs; CTA load max (\d+) mean ([\d.]+) "
+                 r"\(max/mean ([\d.]+)\); largest unit (\d+); host ([\d.]+) us", lines[-1])
+    assert m, lines[-1]
+    assert int(m.group(1)) == n and int(m.group(2)) == n_cta and int(m.group(3)) == mx
+    assert abs(float(m.group(4)) - total / n_cta) < 0.05 and int(m.group(6)) == biggest
+    env["OPATTN_LOG"] = "0"
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, check=True)
+    assert "opattn:" not in r.stderr
