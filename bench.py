@@ -29,6 +29,7 @@ work over that time.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import math
 import os
@@ -201,6 +202,64 @@ def oracle_sample(w, q, k, v, seconds: float, seed: int = 0):
     return {"flops": done_flops, "seconds": t_total, "rows": done_rows, "threads": threads}
 
 
+def host_time_us(fn, reps: int, torch, dev) -> float:
+    """Median host time of fn() in microseconds, each call made with the GPU idle
+    (synchronized before the call; the call itself is not waited for)."""
+    ts = []
+    for _ in range(reps):
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter_ns()
+        fn()
+        ts.append((time.perf_counter_ns() - t0) / 1e3)
+    torch.cuda.synchronize(dev)
+    return statistics.median(ts)
+
+
+def copy_ceiling(pairs_in, pairs_out, steps: int, flops: int, torch, dev):
+    """Rates of the e2e loop's copies alone, one cudaMemcpyAsync per tensor as the loop
+    issues them: host->device only, device->host only, and both directions at once on
+    two streams.  Returns the dict of the bench line's e2e.copy_ceiling."""
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    b_in = sum(d.numel() * d.element_size() for d, _ in pairs_in)
+    b_out = sum(h.numel() * h.element_size() for h, _ in pairs_out)
+
+    def timed(do_in, do_out):
+        for _ in range(2):  # warm
+            with torch.cuda.stream(s_in):
+                for d, h in (pairs_in if do_in else []):
+                    d.copy_(h, non_blocking=True)
+            with torch.cuda.stream(s_out):
+                for h, d in (pairs_out if do_out else []):
+                    h.copy_(d, non_blocking=True)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        cur = torch.cuda.current_stream(dev)
+        e0.record(cur)
+        s_in.wait_event(e0)
+        s_out.wait_event(e0)
+        for _ in range(steps):
+            with torch.cuda.stream(s_in):
+                for d, h in (pairs_in if do_in else []):
+                    d.copy_(h, non_blocking=True)
+            with torch.cuda.stream(s_out):
+                for h, d in (pairs_out if do_out else []):
+                    h.copy_(d, non_blocking=True)
+        cur.wait_stream(s_in)
+        cur.wait_stream(s_out)
+        e1.record(cur)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / steps  # ms per step
+
+    ms_in = timed(True, False)
+    ms_out = timed(False, True)
+    ms_both = timed(True, True)
+    return {"steps": steps, "h2d_gbs": b_in / ms_in / 1e6, "d2h_gbs": b_out / ms_out / 1e6,
+            "both_ms_per_step": ms_both, "both_gbs": (b_in + b_out) / ms_both / 1e6,
+            "ceiling_value": flops / (ms_both / 1e3) / 1e12,
+            "how": "the e2e loop's own tensors, one cudaMemcpyAsync per tensor; 'both' runs the H2D and D2H "
+                   "streams concurrently, ceiling_value = FLOPs per step / both_ms_per_step"}
+
+
 # ----------------------------------------------------------- reference arm
 
 REFERENCE_BUDGET_S = 150.0  # host time of the reference arm's timed steps
@@ -332,6 +391,29 @@ def run_ours(args, w):
     kernel_ms = statistics.mean(launch_ms)
     achieved = flops / (kernel_ms / 1e3) / 1e12
 
+    # Sustained: back-to-back plan runs for a fixed duration (the board settles at its
+    # power cap), with the clocks sampled over that stretch; compared with the measured
+    # sustained GEMM peak.
+    sustained = None
+    if args.sustained_seconds > 0:
+        n_sus = max(args.steps, int(math.ceil(args.sustained_seconds / (kernel_ms / 1e3))))
+        sampler2 = ClockSampler(gpu_selector(torch, local))
+        sampler2.start()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(n_sus):
+            run_plan()
+        s1.record(stream)
+        torch.cuda.synchronize(dev)
+        clocks_sus = sampler2.stop()
+        sus_s, sus_flops = aggregate_over_ranks(s0.elapsed_time(s1) / 1e3, float(flops) * n_sus,
+                                                dist if world > 1 else None)
+        sustained = {"launches": n_sus, "seconds": sus_s, "value": sus_flops / sus_s / 1e12, "unit": "TFLOP/s",
+                     "clocks": clocks_sus}
+
     # End to end through the one-shot C-ABI call with pinned host buffers.  Every
     # step copies its inputs host -> device, runs the call and copies O and LSE
     # back, all inside the timed region.  Two device buffer sets and separate
@@ -398,6 +480,40 @@ def run_ours(args, w):
     e2e_value = e2e_flops / e2e_elapsed / 1e12
     h2d = q.numel() * 2 + k.numel() * 2 + v.numel() * 2  # for a paged cache: the whole cache
     d2h = o.numel() * 2 + lse.numel() * 4
+    ceiling = copy_ceiling([(dq[0], hq), (dk[0], hk), (dv[0], hv)], [(ho[0], do[0]), (hl[0], dl[0])],
+                           min(e2e_steps, 50), flops, torch, dev)
+
+    # Host time of the one-shot call (validation, schedule, staging, launches) with the GPU
+    # idle, beside the scheduler alone and the cost of a ctypes call that does nothing.
+    lib = pkg.load()
+    host = None
+    if not paged:
+        cq_np = np.ascontiguousarray(w.cu_q, dtype=np.int32)
+        ck_np = np.ascontiguousarray(w.cu_k, dtype=np.int32)
+        cq_p, ck_p = cq_np.ctypes.data, ck_np.ctypes.data
+        entry = lib.opattn_decode if decode else lib.opattn_prefill
+        raw_args = (dq[0].data_ptr(), dk[0].data_ptr(), dv[0].data_ptr(), do[0].data_ptr(), dl[0].data_ptr(),
+                    cq_p, ck_p, w.n_seq, w.Hq, w.Hkv, w.d, w.scale, stream.cuda_stream)
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        n_units_c, n_used_c = ctypes.c_int64(0), ctypes.c_int32(0)
+        sched = lib.opattn_decode_schedule_default if decode else lib.opattn_schedule
+        sched(cq_p, ck_p, w.n_seq, w.Hq, w.Hkv, w.d, sms, None, 0, None, ctypes.byref(n_units_c),
+              ctypes.byref(n_used_c))
+        width = len(pkg.DEC_UNIT_FIELDS if decode else pkg.UNIT_FIELDS)
+        u_buf = np.zeros((max(1, n_units_c.value), width), dtype=np.int32)
+        o_buf = np.zeros(sms + 1, dtype=np.int32)
+        u_p, o_p = u_buf.ctypes.data, o_buf.ctypes.data
+        host = {
+            "us_per_call": host_time_us(lambda: entry(*raw_args), 60, torch, dev),
+            "schedule_us": host_time_us(lambda: sched(cq_p, ck_p, w.n_seq, w.Hq, w.Hkv, w.d, sms, u_p,
+                                                      u_buf.shape[0], o_p, ctypes.byref(n_units_c),
+                                                      ctypes.byref(n_used_c)), 60, torch, dev),
+            "ffi_us": host_time_us(lib.opattn_version, 60, torch, dev),
+            "kernel_us": kernel_ms * 1e3,
+            "how": "median of 60 calls with the GPU idle: us_per_call = the one-shot C call (validation, "
+                   "schedule, staging, upload and attention launches); schedule_us = the host scheduler "
+                   "alone; ffi_us = a ctypes call that does nothing",
+        }
     plan.close()
 
     cpu_base = None
@@ -439,7 +555,13 @@ def run_ours(args, w):
             "roofline": roofline,
             "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "steps": e2e_steps, "pipelined": "three buffer sets; copies overlap the neighbouring steps",
-                    "gpu_launches": 2 * e2e_steps},  # per one-shot call: the work-list upload and the attention kernel
+                    "gpu_launches": 2 * e2e_steps,  # per one-shot call: the work-list upload and the attention kernel
+                    "copy_ceiling": ceiling},
+            "host_us_per_call": host["us_per_call"] if host else None,
+            "host": host,
+            "sustained": (dict(sustained, frac=sustained["value"] / peak_sus,
+                               peak=peak_sus, peak_source=f"{peak_src} bf16_tflops_sustained")
+                          if sustained and not decode else sustained),
             "cpu_baseline": cpu_base,
             "clocks": clocks,
             "gpu_launches": args.steps,
@@ -495,6 +617,8 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=0,
                     help="steps of the end-to-end measurement (default 0: as many as --steps)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--sustained-seconds", type=float, default=3.0,
+                    help="duration of the back-to-back 'sustained' measurement (0: skip)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--reference-step-seconds", type=float, default=3.0,
                     help="oracle time per reference step, capped so that all steps take about "
