@@ -612,7 +612,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama3_70b",
-                    help="tiny | llama3_8b | llama3_70b | bursty | chunked | decode_llama3_70b | "
+                    help="tiny | llama3_8b | llama3_70b | bursty | chunked | chunk_long_prefix | "
+                         "chunks_long_prefix | decode_llama3_70b | "
                          "decode_llama3_8b | decode_spec4_llama3_70b | decode_llama3_70b_paged16")
     ap.add_argument("--e2e-steps", type=int, default=0,
                     help="steps of the end-to-end measurement (default 0: as many as --steps)")
@@ -625,7 +626,7 @@ def main(argv=None):
                          f"{REFERENCE_BUDGET_S:.0f} s")
     args = ap.parse_args(argv)
     from paper_2608_13499_gb300 import workloads as W
-    w = {**W.STANDARD, **W.DECODE}[args.workload]()
+    w = {**W.STANDARD, **W.LONG_PREFIX, **W.DECODE}[args.workload]()
     if args.impl == "reference":
         return run_reference(args, w)
     return run_ours(args, w)

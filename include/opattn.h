@@ -80,8 +80,13 @@ OPATTN_API const char *opattn_status_string(int32_t status);
  * list on the host (L2-sized groups of (sequence, kv head) pairs, longest
  * unit first within a group) in mapped pinned memory, then launches on
  * `stream` a small upload kernel that reads it into stream-ordered device
- * scratch (cudaMallocAsync / cudaFreeAsync) and one persistent kernel over
- * min(#SMs, #units) CTAs; no copy-engine transfer.  Returns OPATTN_OK with no
+ * scratch and one persistent kernel over min(#SMs, #units) CTAs (or, for a
+ * batch split into pieces, one CTA per SM); no copy-engine transfer.  The
+ * scratch (the work list, and the pieces' partial results when key ranges
+ * are split: 129 fp32 per row of a piece at d = 128) is allocated with
+ * cudaMallocFromPoolAsync from a memory pool the library creates per device
+ * and freed on `stream`; the pool keeps up to 64 MB of freed scratch mapped
+ * between calls.  Returns OPATTN_OK with no
  * device work when total_q == 0.  `scale` must be finite and > 0 (usually
  * 1 / sqrt(d)).  Device-side wait timeouts are not reported here; use
  * opattn_prefill_checked to observe them.
@@ -100,8 +105,11 @@ OPATTN_API opattn_status opattn_prefill(const void *q, const void *k, const void
  * stream-ordered allocator.  Same arguments and computation as
  * opattn_prefill; the caller still provides q, k, v, o and lse.  The work
  * list and status word go to a fixed device array inside the library
- * (OPATTN_NOALLOC_MAX_UNITS work units of 32 bytes plus 8 KiB, about 1 MiB),
- * which every GPU that loads the library keeps until the process exits.  It
+ * (OPATTN_NOALLOC_MAX_UNITS work units of 52 bytes plus 8 KiB, about
+ * 1.7 MB), which every GPU that loads the library keeps until the process
+ * exits.  Key ranges are never split here (the array has no room for the
+ * pieces' partial results), so a batch that opattn_prefill would split runs
+ * as the list schedule and agrees with it within the tolerance only.  It
  * calls no cudaMalloc, cudaMallocAsync or cudaFree, and no cudaHostAlloc
  * either: the host side builds the list in ordinary heap memory and copies
  * it with cudaMemcpyAsync.
@@ -180,20 +188,32 @@ OPATTN_API opattn_status opattn_plan_info(const opattn_plan *plan, int64_t *n_un
 
 /*
  * Host-only scheduler (no GPU needed), exposed for testing and capacity
- * planning.  A work unit is (sequence, kv head, block of 2 * (128 / G)
- * query tokens).  Its cost is the number of 128-key tiles it visits after
- * whole tiles above the causal diagonal are skipped, plus one.  The
- * (sequence, kv head) pairs are gathered in order into groups of at most
- * 48 MB of K/V (so that a group's K/V stays in L2); units are taken group by
- * group, longest first within a group, and each is given to the CTA with the
- * least assigned cost so far (greedy list scheduling: makespan within the
- * mean load plus the largest unit).  A CTA runs its units in that order.
- * Writes `units` as 8 int32 per unit:
+ * planning: the work list opattn_prefill and opattn_plan_create build.  A
+ * work unit is (sequence, kv head, block of 2 * (128 / G) query tokens).
+ * Its cost is the number of 128-key tiles it visits after whole tiles above
+ * the causal diagonal are skipped, plus one.  The (sequence, kv head) pairs
+ * are gathered in order into groups of at most 48 MB of K/V (so that a
+ * group's K/V stays in L2); units are taken group by group, longest first
+ * within a group, and each is given to the CTA with the least assigned cost
+ * so far (greedy list scheduling: makespan within the mean load plus the
+ * largest unit).  A CTA runs its units in that order.
+ * Split-KV: when the largest units set that makespan (few units over long
+ * key ranges, e.g. one prompt chunk over a long cached prefix), the key
+ * tiles of all units, in pair order, are instead cut into one equal stretch
+ * per CTA; a unit cut by stretch boundaries becomes pieces on consecutive
+ * CTAs, each over its own run of key tiles, whose partial results the last
+ * piece to finish merges in the same launch.  The cut is taken when a
+ * CTA's stretch is at least 4 key tiles and its makespan, counting two more
+ * per piece, is below 0.85 of the list schedule's.
+ * Writes `units` as 13 int32 per unit (or piece):
  *     {first packed query row, tokens in unit, first packed key row of the
  *      sequence, Lk, last visible key of the unit's first token, kv head,
- *      key tiles visited, sequence index}
+ *      key tiles visited, sequence index, first key tile visited, partial
+ *      slot (-1: not split), merge group (-1: not split), piece index,
+ *      pieces of the unit}
  * grouped by CTA, and cta_offsets[0..n_ctas] (unit index ranges).  n_ctas
- * used = min(n_ctas, #units), returned in *n_ctas_used.  Fails with
+ * used = min(n_ctas, #units) for the list schedule and min(n_ctas, key
+ * tiles) for the cut, returned in *n_ctas_used.  Fails with
  * OPATTN_ERR_CAPACITY (and *n_units_out set) if unit_capacity is too small.
  */
 OPATTN_API opattn_status opattn_schedule(const int32_t *cu_seqlens_q, const int32_t *cu_seqlens_k,
@@ -219,8 +239,8 @@ OPATTN_API opattn_status opattn_schedule(const int32_t *cu_seqlens_q, const int3
  * work.  Lk may be anything, including 0 and Lk < Lq.
  *
  * Scratch: the one-shot call allocates its work list and the chunks'
- * partial results (kDecCols x d fp32 per chunk, 16 KB) with cudaMallocAsync
- * on `stream` and frees them there.  opattn_decode_checked additionally
+ * partial results (kDecCols x d fp32 per chunk, 16 KB) on `stream` from the
+ * library's memory pool (as opattn_prefill) and frees them there.  opattn_decode_checked additionally
  * waits for the stream and reports a device timeout (flags as for
  * opattn_prefill_checked).
  */

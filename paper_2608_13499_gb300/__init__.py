@@ -27,7 +27,8 @@ OPATTN_FLAG_TEST_FORCE_TIMEOUT = 1
 OPATTN_FLAG_TEST_FORCE_TIMEOUT_FIRST_CTA = 2
 OPATTN_NOALLOC_MAX_UNITS = 32768
 
-UNIT_FIELDS = ("q_tok0", "n_tok", "k_row0", "Lk", "qlim0", "kvh", "n_tiles", "seq")
+UNIT_FIELDS = ("q_tok0", "n_tok", "k_row0", "Lk", "qlim0", "kvh", "n_tiles", "seq", "tile0", "part", "group", "chunk",
+               "n_chunks")
 DEC_UNIT_FIELDS = ("q_tok0", "nq", "k_row0", "Lk", "kvh", "tile0", "n_tiles", "part", "group", "chunk", "n_chunks",
                    "seq")
 DEC_COLS = 32
@@ -154,7 +155,7 @@ def opattn_prefill(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: int, Hq: 
 def opattn_prefill_noalloc(q, k, v, o, lse, cu_seqlens_q, cu_seqlens_k, n_seq: int, Hq: int, Hkv: int, d: int,
                            scale: float, stream=None, *, check: bool = True) -> int:
     """C ``opattn_prefill_noalloc``: same arguments as opattn_prefill, but the library
-    allocates no device memory (its work list goes to a fixed ~1 MiB device array
+    allocates no device memory (its work list goes to a fixed ~1.7 MB device array
     shared by all calls; see include/opattn.h).  For callers that cannot let a
     library allocate, e.g. an engine that has reserved nearly all HBM for its own
     pool.  Calls that overlap on the GPU race on the shared array."""
@@ -196,7 +197,7 @@ def _schedule(fn_name: str, width: int, cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv
 
 
 def opattn_schedule(cu_seqlens_q, cu_seqlens_k, Hq: int, Hkv: int, d: int, n_ctas: int):
-    """C ``opattn_schedule`` (host only).  Returns (units [n, 8] int32, cta_offsets [n_ctas_used + 1])."""
+    """C ``opattn_schedule`` (host only).  Returns (units [n, 13] int32, cta_offsets [n_ctas_used + 1])."""
     return _schedule("opattn_schedule", len(UNIT_FIELDS), cu_seqlens_q, cu_seqlens_k, Hq, Hkv, d, n_ctas)
 
 

@@ -75,9 +75,11 @@ opattn_status check_tensors(const void* q, const void* k, const void* v, const v
 // ------------------------------------------------------------- scheduler
 
 struct Schedule {
-    std::vector<UnitRec> units;    // grouped by CTA, longest first within a CTA
+    std::vector<UnitRec> units;    // grouped by CTA, in the order each CTA runs them
     std::vector<int32_t> cta_off;  // n_cta + 1
     int32_t n_cta = 0;
+    int32_t n_groups = 0;          // split units (kUnitWarps merge counters each)
+    int32_t n_parts = 0;           // pieces of split units (one partial slot each)
 };
 
 // K/V bytes of the (sequence, kv head) pairs whose units run together: small
@@ -95,10 +97,12 @@ constexpr int64_t kL2GroupBytes = 48ll << 20;
 // the lowest CTA index at that load, which is the order of (load, index)
 // pairs.  Batches whose buckets would take more than kMaxBucketWords words
 // use a heap of (load, index) pairs instead.
+// The units are taken in the order order[0], order[1], ... (indices into `all`).
 template <class U, class CostFn>
-void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std::vector<U>* units,
-               std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
-    const int64_t n = static_cast<int64_t>(ordered.size());
+void list_pack(const std::vector<U>& all, const std::vector<uint32_t>& order, int32_t max_ctas, CostFn cost,
+               std::vector<U>* units, std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
+    auto ordered = [&](int64_t i) -> const U& { return all[order[static_cast<size_t>(i)]]; };
+    const int64_t n = static_cast<int64_t>(order.size());
     units->clear();
     cta_off->clear();
     *n_cta_out = 0;
@@ -107,7 +111,7 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
     std::vector<int32_t> owner(static_cast<size_t>(n));
     std::vector<int32_t> per_cta(static_cast<size_t>(n_cta), 0);
     int64_t max_cost = 1;
-    for (const U& u : ordered) max_cost = std::max<int64_t>(max_cost, cost(u));
+    for (int64_t i = 0; i < n; ++i) max_cost = std::max<int64_t>(max_cost, cost(ordered(i)));
     const size_t words = (static_cast<size_t>(n_cta) + 63) / 64;
     constexpr size_t kMaxBucketWords = size_t{1} << 20;
     const size_t n_buckets = static_cast<size_t>(max_cost) + 1;
@@ -132,7 +136,7 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
             --count[b];
             owner[static_cast<size_t>(i)] = c;
             ++per_cta[static_cast<size_t>(c)];
-            const int64_t nl = load[static_cast<size_t>(c)] + cost(ordered[static_cast<size_t>(i)]);
+            const int64_t nl = load[static_cast<size_t>(c)] + cost(ordered(i));
             load[static_cast<size_t>(c)] = nl;
             const size_t nb = static_cast<size_t>(nl % static_cast<int64_t>(n_buckets));
             bits[nb * words + (static_cast<size_t>(c) >> 6)] |= uint64_t{1} << (c & 63);
@@ -147,7 +151,7 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
             heap.pop();
             owner[static_cast<size_t>(i)] = sl.second;
             ++per_cta[static_cast<size_t>(sl.second)];
-            sl.first += cost(ordered[static_cast<size_t>(i)]);
+            sl.first += cost(ordered(i));
             heap.push(sl);
         }
     }
@@ -158,9 +162,116 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
     units->resize(static_cast<size_t>(n));
     for (int64_t i = 0; i < n; ++i) {
         const int32_t c = owner[static_cast<size_t>(i)];
-        (*units)[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = ordered[static_cast<size_t>(i)];
+        (*units)[static_cast<size_t>(fill[static_cast<size_t>(c)]++)] = ordered(i);
     }
     *n_cta_out = n_cta;
+}
+
+// Split-KV for units over long key ranges.  When a batch has few units for
+// the grid (one prompt chunk over a long cached prefix, say), the longest
+// unit sets the list schedule's makespan however the rest are placed.  The
+// stream-K cut takes the key tiles of all units in pair order and cuts them
+// into one equal stretch per CTA; a unit that falls into several stretches
+// becomes pieces on consecutive CTAs, each over its own run of key tiles,
+// and the piece that finishes last merges the pieces' partial results.  A
+// piece costs its tiles, one for its Q load and epilogue, and one more for
+// writing its partial result and its share of the merge.
+constexpr int64_t kPieceOverhead = 2;
+// The cut replaces the list schedule only when its makespan (in those costs)
+// is below this fraction of the list schedule's, and only when a CTA's
+// stretch is at least kMinStretchTiles key tiles: below that the batch is
+// small enough that launch and load latency, not the makespan, set its time.
+constexpr double kSplitGain = 0.85;
+constexpr int64_t kMinStretchTiles = 4;
+
+int64_t max_cta_load(const std::vector<UnitRec>& units, const std::vector<int32_t>& cta_off) {
+    int64_t mx = 0;
+    for (size_t c = 0; c + 1 < cta_off.size(); ++c) {
+        int64_t load = 0;
+        for (int32_t i = cta_off[c]; i < cta_off[c + 1]; ++i) {
+            const UnitRec& u = units[static_cast<size_t>(i)];
+            load += u.n_tiles + 1 + (u.part >= 0 ? kPieceOverhead : 0);
+        }
+        mx = std::max(mx, load);
+    }
+    return mx;
+}
+
+// The stream-K cut of `all` (units in pair order) over at most max_ctas CTAs.
+// Units without key tiles are spread over the CTAs round robin.
+void stream_k_prefill(const std::vector<UnitRec>& all, int32_t max_ctas, Schedule* out) {
+    int64_t total = 0;
+    for (const UnitRec& u : all) total += u.n_tiles;
+    out->units.clear();
+    out->cta_off.clear();
+    out->n_groups = 0;
+    out->n_parts = 0;
+    const int32_t n_cta = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(max_ctas, total)));
+    std::vector<std::vector<UnitRec>> per_cta(static_cast<size_t>(n_cta));
+    auto bound = [&](int64_t c) { return c * total / n_cta; };  // first tile of CTA c's stretch
+    int64_t pos = 0;
+    int32_t rr = 0;
+    for (const UnitRec& u : all) {
+        if (u.n_tiles <= 0) {
+            per_cta[static_cast<size_t>(rr)].push_back(u);
+            rr = (rr + 1) % n_cta;
+            continue;
+        }
+        int64_t c = std::min<int64_t>(n_cta - 1, pos * n_cta / total);
+        while (c > 0 && bound(c) > pos) --c;
+        while (c + 1 < n_cta && bound(c + 1) <= pos) ++c;
+        const int64_t end = pos + u.n_tiles;
+        std::vector<std::array<int64_t, 3>> pieces;  // (CTA, first tile, tiles)
+        for (int64_t t = pos; t < end; ++c) {
+            const int64_t stop = std::min<int64_t>(end, bound(c + 1));
+            if (stop > t) pieces.push_back({c, t - pos, stop - t});
+            t = stop;
+        }
+        const int32_t k = static_cast<int32_t>(pieces.size());
+        for (int32_t i = 0; i < k; ++i) {
+            UnitRec p = u;
+            p.tile0 = static_cast<int32_t>(pieces[static_cast<size_t>(i)][1]);
+            p.n_tiles = static_cast<int32_t>(pieces[static_cast<size_t>(i)][2]);
+            p.part = k > 1 ? out->n_parts + i : -1;
+            p.group = k > 1 ? out->n_groups : -1;
+            p.chunk = i;
+            p.n_chunks = k;
+            per_cta[static_cast<size_t>(pieces[static_cast<size_t>(i)][0])].push_back(p);
+        }
+        if (k > 1) {
+            out->n_parts += k;
+            ++out->n_groups;
+        }
+        pos = end;
+    }
+    out->cta_off.assign(static_cast<size_t>(n_cta) + 1, 0);
+    for (int32_t c = 0; c < n_cta; ++c) {
+        const auto& v = per_cta[static_cast<size_t>(c)];
+        out->cta_off[static_cast<size_t>(c) + 1] = out->cta_off[static_cast<size_t>(c)] + static_cast<int32_t>(v.size());
+        out->units.insert(out->units.end(), v.begin(), v.end());
+    }
+    out->n_cta = n_cta;
+}
+
+// Replaces the list schedule in `out` by the stream-K cut of `all` when the
+// cut's makespan is below kSplitGain of the list schedule's.  A quick bound
+// first: the cut cannot beat mean load + 2 pieces' overhead, so batches whose
+// list schedule is already within that are left alone.
+void split_if_faster(const std::vector<UnitRec>& all, int32_t max_ctas, Schedule* out) {
+    if (out->n_cta <= 0 || all.empty()) return;
+    int64_t total = 0, tiles = 0;
+    for (const UnitRec& u : all) {
+        total += u.n_tiles + 1;
+        tiles += u.n_tiles;
+    }
+    const int32_t cap = std::max<int32_t>(max_ctas, 1);
+    if (tiles < kMinStretchTiles * cap) return;
+    const int64_t lpt = max_cta_load(out->units, out->cta_off);
+    const double floor = static_cast<double>(total) / cap;
+    if (static_cast<double>(lpt) * kSplitGain <= floor) return;
+    Schedule sk;
+    stream_k_prefill(all, cap, &sk);
+    if (static_cast<double>(max_cta_load(sk.units, sk.cta_off)) < kSplitGain * static_cast<double>(lpt)) *out = sk;
 }
 
 // Units are (sequence, kv head, block of 2 * TPB query tokens).  Cost is the
@@ -174,7 +285,8 @@ void list_pack(const std::vector<U>& ordered, int32_t max_ctas, CostFn cost, std
 // assignment keeps the makespan within mean load + largest unit.  The
 // longest-first order within a group is a stable counting sort on the tile
 // count (O(units + tiles) per group).
-void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out) {
+void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out,
+                    bool allow_split = true) {
     const int32_t tpu = 2 * g.TPB;
     int64_t n_units = 0;
     for (int32_t s = 0; s < g.n_seq; ++s) n_units += (static_cast<int64_t>(cu_q[s + 1] - cu_q[s]) + tpu - 1) / tpu;
@@ -208,6 +320,11 @@ void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g,
             u.kvh = 0;
             u.n_tiles = n_tiles;
             u.seq = s;
+            u.tile0 = 0;
+            u.part = -1;
+            u.group = -1;
+            u.chunk = 0;
+            u.n_chunks = 1;
         }
         const size_t per_head = n - first;
         const int64_t pair_bytes = static_cast<int64_t>(Lk) * pair_row_bytes;
@@ -226,8 +343,8 @@ void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g,
         }
         n = first + static_cast<size_t>(g.Hkv) * per_head;
     }
-    // group by group, longest first within a group (stable counting sort)
-    std::vector<UnitRec> ordered(all.size());
+    // group by group, longest first within a group (stable counting sort of indices)
+    std::vector<uint32_t> order(all.size());
     std::vector<size_t> slot;
     group_start.push_back(all.size());
     for (size_t gi = 0; gi + 1 < group_start.size(); ++gi) {
@@ -237,23 +354,35 @@ void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g,
         for (size_t i = b; i < e; ++i) ++slot[static_cast<size_t>(mx - all[i].n_tiles) + 1];  // rank 0 = most tiles
         slot[0] = b;
         for (size_t r = 1; r < slot.size(); ++r) slot[r] += slot[r - 1];
-        for (size_t i = b; i < e; ++i) ordered[slot[static_cast<size_t>(mx - all[i].n_tiles)]++] = all[i];
+        for (size_t i = b; i < e; ++i) order[slot[static_cast<size_t>(mx - all[i].n_tiles)]++] = static_cast<uint32_t>(i);
     }
-    list_pack(ordered, max_ctas, [](const UnitRec& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
+    list_pack(all, order, max_ctas, [](const UnitRec& u) { return u.n_tiles + 1; }, &out->units, &out->cta_off,
               &out->n_cta);
+    out->n_groups = 0;
+    out->n_parts = 0;
+    if (allow_split) split_if_faster(all, max_ctas, out);
 }
 
-// Device work area: [cta_off (n_cta + 1) | pad to 32 B | units | status].
+// Device work area: [cta_off (n_cta + 1) | pad to 32 B | units | merge
+// counters (kUnitWarps per split unit, 8 bytes each) | run words | status |
+// pad 256 | part_lse (n_parts x kUnitRows fp32) | part_o (n_parts x
+// kUnitRows x d fp32)].  The counters, run words and status word are
+// contiguous: the one-shot calls zero them with the work-list upload, a plan
+// once when it is created (the counters carry the launch epoch, RunWords).
 struct WorkLayout {
-    size_t off_units, off_status, bytes, upload_bytes;
+    size_t off_units, off_counters, off_run, off_status, off_part_lse, off_part_o, bytes, upload_bytes, zero_bytes;
 };
-WorkLayout work_layout(const Schedule& s) {
+WorkLayout work_layout(const Schedule& s, int32_t d) {
     WorkLayout w;
-    const size_t off_bytes = (s.cta_off.size() * sizeof(int32_t) + 31) / 32 * 32;
-    w.off_units = off_bytes;
-    w.off_status = off_bytes + s.units.size() * sizeof(UnitRec);
-    w.upload_bytes = w.off_status;
-    w.bytes = w.off_status + 32;
+    w.off_units = (s.cta_off.size() * sizeof(int32_t) + 31) / 32 * 32;
+    w.off_counters = (w.off_units + s.units.size() * sizeof(UnitRec) + 15) / 16 * 16;
+    w.off_run = w.off_counters + static_cast<size_t>(s.n_groups) * kUnitWarps * sizeof(unsigned long long);
+    w.off_status = w.off_run + sizeof(RunWords);
+    w.upload_bytes = w.off_counters;
+    w.zero_bytes = w.off_status + sizeof(int32_t) - w.off_counters;
+    w.off_part_lse = (w.off_status + sizeof(int32_t) + 255) / 256 * 256;
+    w.off_part_o = w.off_part_lse + (static_cast<size_t>(s.n_parts) * kUnitRows * sizeof(float) + 255) / 256 * 256;
+    w.bytes = w.off_part_o + static_cast<size_t>(s.n_parts) * kUnitRows * static_cast<size_t>(d) * sizeof(float);
     return w;
 }
 void pack_upload(const Schedule& s, const WorkLayout& w, uint8_t* dst) {
@@ -372,6 +501,52 @@ bool upload_staged(const Staging* s, void* dst, size_t bytes, void* zero, size_t
            cudaMemsetAsync(zero, 0, zero_bytes, stream) == cudaSuccess;
 }
 
+// Stream-ordered scratch of the one-shot calls comes from a memory pool the
+// library creates per device.  It keeps up to kPoolKeepBytes of freed scratch
+// mapped across synchronizations, where the device's default pool (release
+// threshold 0 unless its owner raises it) hands freed memory back to the
+// system at every synchronization and maps it again on the next call.  If
+// the pool cannot be created the default pool serves the calls.
+constexpr uint64_t kPoolKeepBytes = 64ull << 20;
+constexpr int kMaxPoolDevices = 64;
+
+cudaMemPool_t scratch_pool() {
+    static std::mutex mu;
+    static cudaMemPool_t pools[kMaxPoolDevices] = {};
+    static bool tried[kMaxPoolDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxPoolDevices) {
+        (void)cudaGetLastError();
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lk(mu);
+    if (!tried[dev]) {
+        tried[dev] = true;
+        cudaMemPoolProps props;
+        std::memset(&props, 0, sizeof props);
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        cudaMemPool_t pool = nullptr;
+        if (cudaMemPoolCreate(&pool, &props) == cudaSuccess) {
+            uint64_t keep = kPoolKeepBytes;
+            if (cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep) == cudaSuccess) {
+                pools[dev] = pool;
+            } else {
+                cudaMemPoolDestroy(pool);
+            }
+        }
+        (void)cudaGetLastError();
+    }
+    return pools[dev];
+}
+
+// cudaMallocAsync from the library's pool (or the default pool).
+cudaError_t scratch_alloc(void** ptr, size_t bytes, cudaStream_t stream) {
+    cudaMemPool_t pool = scratch_pool();
+    return pool ? cudaMallocFromPoolAsync(ptr, bytes, pool, stream) : cudaMallocAsync(ptr, bytes, stream);
+}
+
 int device_sm_count() {
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
@@ -380,7 +555,8 @@ int device_sm_count() {
 }
 
 LaunchArgs make_args(const void* q, const void* k, const void* v, void* o, float* lse, const Geometry& g,
-                     float scale, const uint8_t* work, const WorkLayout& w, int32_t n_cta, uint32_t flags) {
+                     float scale, const uint8_t* work, const WorkLayout& w, const Schedule& sch, uint32_t flags) {
+    const int32_t n_cta = sch.n_cta;
     LaunchArgs a;
     a.q = q;
     a.k = k;
@@ -398,6 +574,13 @@ LaunchArgs make_args(const void* q, const void* k, const void* v, void* o, float
     a.n_cta = n_cta;
     a.status = reinterpret_cast<int32_t*>(const_cast<uint8_t*>(work) + w.off_status);
     a.flags = flags;
+    if (sch.n_groups > 0) {
+        uint8_t* wb = const_cast<uint8_t*>(work);
+        a.counters = reinterpret_cast<unsigned long long*>(wb + w.off_counters);
+        a.run = reinterpret_cast<RunWords*>(wb + w.off_run);
+        a.part_lse = reinterpret_cast<float*>(wb + w.off_part_lse);
+        a.part_o = reinterpret_cast<float*>(wb + w.off_part_o);
+    }
     return a;
 }
 
@@ -467,22 +650,22 @@ opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o,
     Schedule sch;
     build_schedule(cu_q, cu_k, g, sms, &sch);
     log_schedule("prefill", sch.units, sch.cta_off, prefill_cost, us_since(t_entry));
-    const WorkLayout w = work_layout(sch);
+    const WorkLayout w = work_layout(sch, g.d);
     Staging* stg = staging_acquire(w.upload_bytes);
     if (!stg) return OPATTN_ERR_CUDA;
     pack_upload(sch, w, static_cast<uint8_t*>(stg->host));
 
     void* work = nullptr;
-    if (cudaMallocAsync(&work, w.bytes, stream) != cudaSuccess) {
+    if (scratch_alloc(&work, w.bytes, stream) != cudaSuccess) {
         staging_release(stg, stream);
         return OPATTN_ERR_CUDA;
     }
-    bool ok = upload_staged(stg, work, w.upload_bytes, static_cast<uint8_t*>(work) + w.off_status, sizeof(int32_t),
+    bool ok = upload_staged(stg, work, w.upload_bytes, static_cast<uint8_t*>(work) + w.off_counters, w.zero_bytes,
                             stream);
     staging_release(stg, stream);
     int32_t dev_status = 0;
     if (ok) {
-        LaunchArgs a = make_args(q, k, v, o, lse, g, scale, static_cast<uint8_t*>(work), w, sch.n_cta, flags);
+        LaunchArgs a = make_args(q, k, v, o, lse, g, scale, static_cast<uint8_t*>(work), w, sch, flags);
         if (paged) {
             a.block_table = paged->block_table;
             a.max_blocks = paged->max_blocks;
@@ -539,9 +722,10 @@ opattn_status prefill_noalloc_impl(const void* q, const void* k, const void* v, 
     if (sms <= 0) return OPATTN_ERR_CUDA;
 
     Schedule sch;
-    build_schedule(cu_q, cu_k, g, std::min(sms, kNoAllocMaxCtas), &sch);
+    // No split-KV here: the fixed array has no room for the pieces' partials.
+    build_schedule(cu_q, cu_k, g, std::min(sms, kNoAllocMaxCtas), &sch, /*allow_split=*/false);
     log_schedule("prefill (no-alloc)", sch.units, sch.cta_off, prefill_cost, us_since(t_entry));
-    const WorkLayout w = work_layout(sch);
+    const WorkLayout w = work_layout(sch, g.d);
     void* scratch = nullptr;
     size_t scratch_bytes = 0;
     if (noalloc_scratch(&scratch, &scratch_bytes) != 0) return OPATTN_ERR_CUDA;
@@ -556,7 +740,7 @@ opattn_status prefill_noalloc_impl(const void* q, const void* k, const void* v, 
     // The array keeps the previous call's contents: the status word must
     // start at zero.
     if (cudaMemsetAsync(work + w.off_status, 0, sizeof(int32_t), stream) != cudaSuccess) return OPATTN_ERR_CUDA;
-    const LaunchArgs a = make_args(q, k, v, o, lse, g, scale, work, w, sch.n_cta, 0u);
+    const LaunchArgs a = make_args(q, k, v, o, lse, g, scale, work, w, sch, 0u);
     return launch_prefill(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
 }
 
@@ -885,7 +1069,7 @@ opattn_status decode_impl(const void* q, const void* k, const void* v, void* o, 
     if (!stg) return OPATTN_ERR_CUDA;
     pack_decode_upload(sch, w, static_cast<uint8_t*>(stg->host));
     void* work = nullptr;
-    if (cudaMallocAsync(&work, w.bytes, stream) != cudaSuccess) {
+    if (scratch_alloc(&work, w.bytes, stream) != cudaSuccess) {
         staging_release(stg, stream);
         return OPATTN_ERR_CUDA;
     }
@@ -1001,14 +1185,16 @@ opattn_status opattn_plan_create(opattn_plan** plan, const int32_t* cu_seqlens_q
         const Clock::time_point t0 = Clock::now();
         build_schedule(cu_seqlens_q, cu_seqlens_k, g, cap, &p->sch);
         log_schedule("prefill plan", p->sch.units, p->sch.cta_off, prefill_cost, us_since(t0));
-        p->w = work_layout(p->sch);
-        std::vector<uint8_t> host(p->w.bytes, 0);
+        p->w = work_layout(p->sch, g.d);
+        // the work list, then the counters, run words and status word at zero
+        const size_t init_bytes = p->w.off_counters + p->w.zero_bytes;
+        std::vector<uint8_t> host(init_bytes, 0);
         pack_upload(p->sch, p->w, host.data());
         if (cudaMalloc(&p->work, p->w.bytes) != cudaSuccess) {
             delete p;
             return OPATTN_ERR_CUDA;
         }
-        if (cudaMemcpy(p->work, host.data(), p->w.bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+        if (cudaMemcpy(p->work, host.data(), init_bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
             cudaFree(p->work);
             delete p;
             return OPATTN_ERR_CUDA;
@@ -1033,7 +1219,7 @@ opattn_status plan_launch(const opattn_plan* plan, const void* q, const void* k,
                                                     plan->dsch.max_cols, kflags);
         return launch_decode(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
     }
-    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, work, plan->w, plan->sch.n_cta, kflags);
+    const LaunchArgs a = make_args(q, k, v, o, lse, plan->g, scale, work, plan->w, plan->sch, kflags);
     return launch_prefill(a, stream) == 0 ? OPATTN_OK : OPATTN_ERR_CUDA;
 }
 }  // namespace
@@ -1266,7 +1452,7 @@ opattn_status opattn_plan_run_paged(const opattn_plan* plan, const void* q, cons
     uint8_t* work = static_cast<uint8_t*>(plan->work);
     const cudaStream_t st_ = static_cast<cudaStream_t>(stream);
     if (!plan->decode) {
-        LaunchArgs a = make_args(q, k_cache, v_cache, o, lse, plan->g, scale, work, plan->w, plan->sch.n_cta, 0u);
+        LaunchArgs a = make_args(q, k_cache, v_cache, o, lse, plan->g, scale, work, plan->w, plan->sch, 0u);
         a.block_table = block_table;
         a.max_blocks = plan->max_blocks;
         a.block_size = plan->block_size;

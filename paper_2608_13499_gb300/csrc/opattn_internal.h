@@ -11,25 +11,40 @@ namespace opattn {
 // query heads of one kv head (rows ordered token-major, head-minor, which is
 // their order in memory).  A work unit is two M-tiles (2 * TPB tokens) of one
 // sequence and one kv head; each K/V tile of BN keys feeds both M-tiles and
-// all G heads of the group.
+// all G heads of the group.  A unit normally visits every key tile its
+// tokens see; a unit over a long key range may instead be cut into pieces
+// (split-KV) that each cover a stretch of its key tiles on its own CTA and
+// are merged with their log-sum-exp weights by the piece that finishes last.
 constexpr int kRowsPerTile = 128;
 constexpr int kBlockN = 128;
+constexpr int kUnitRows = 2 * kRowsPerTile;  // accumulator rows of a unit
+// Warps of a unit's rows (two M-tiles x four TMEM lane quarters): a split
+// unit has one merge counter per warp.
+constexpr int kUnitWarps = 8;
 
 inline int tokens_per_tile(int G) { return kRowsPerTile / G; }
 inline int tokens_per_unit(int G) { return 2 * tokens_per_tile(G); }
 
-// One work unit; 32 bytes, read by every role of the CTA that owns it.
+// One work unit (or one piece of a split unit); 52 bytes, read field by
+// field by every role of the CTA that owns it (a 16-byte-aligned record read
+// with vector loads keeps every field live and made the kernel spill).
+constexpr int kUnitFields = 13;
 struct UnitRec {
-    int32_t q_tok0;   // packed query row of the unit's first token
-    int32_t n_tok;    // valid tokens in the unit (<= 2 * TPB)
-    int32_t k_row0;   // packed key row of the sequence's first key
-    int32_t Lk;       // keys in the sequence
-    int32_t qlim0;    // last visible key index of the first token (= position + Lk - Lq)
-    int32_t kvh;      // kv head
-    int32_t n_tiles;  // key tiles to visit (0: no row sees a key)
-    int32_t seq;      // sequence index (diagnostics only)
+    int32_t q_tok0;    // packed query row of the unit's first token
+    int32_t n_tok;     // valid tokens in the unit (<= 2 * TPB)
+    int32_t k_row0;    // packed key row of the sequence's first key
+    int32_t Lk;        // keys in the sequence
+    int32_t qlim0;     // last visible key index of the first token (= position + Lk - Lq)
+    int32_t kvh;       // kv head
+    int32_t n_tiles;   // key tiles to visit (0: no row sees a key)
+    int32_t seq;       // sequence index (block-table row of a paged cache)
+    int32_t tile0;     // first key tile visited (0 unless the unit is a later piece of a split unit)
+    int32_t part;      // partial slot of the piece, -1 when the unit is not split
+    int32_t group;     // merge counters of the split unit (kUnitWarps each), -1 when not split
+    int32_t chunk;     // piece index within the unit; its pieces' slots are part - chunk ...
+    int32_t n_chunks;  // pieces of the unit (1 when not split)
 };
-static_assert(sizeof(UnitRec) == 32, "UnitRec must stay 32 bytes");
+static_assert(sizeof(UnitRec) == kUnitFields * 4, "UnitRec must stay 52 bytes");
 
 // Device status word values (written by the kernel's bounded waits).
 constexpr int32_t kDevOk = 0;
@@ -69,6 +84,15 @@ struct LaunchArgs {
     int32_t n_cta;
     int32_t* status;          // device
     uint32_t flags;
+    // Split units (only when the schedule has any, else nullptr): merge
+    // counters (kUnitWarps per split unit), run words, and the pieces'
+    // partial results: part_lse [parts][kUnitRows] (log2 domain) and part_o
+    // [parts][d / 4][kUnitRows][4] fp32 (normalised O, four channels per row
+    // in a 16-byte group so that a warp's 32 rows are 512 contiguous bytes).
+    unsigned long long* counters = nullptr;
+    RunWords* run = nullptr;
+    float* part_lse = nullptr;
+    float* part_o = nullptr;
     // Paged K/V (block_table != nullptr): as in DecodeLaunchArgs.
     const int32_t* block_table = nullptr;
     int32_t max_blocks = 0;

@@ -110,6 +110,11 @@ struct KParams {
     int32_t max_blocks;
     int32_t page_shift;          // log2(page size)
     int32_t o_tma;               // a warp's 32 rows form one TMA box of O (G divides 32, or 32 divides G)
+    // split units (nullptr when the work list has none): see LaunchArgs
+    unsigned long long* counters;
+    RunWords* run;
+    float* part_lse;
+    float* part_o;
 };
 
 template <int D>
@@ -154,7 +159,8 @@ __device__ __forceinline__ void run_producer(const CUtensorMap* tmQ, const CUten
 #pragma unroll
                 for (int b = 0; b < C::kDBlocks; ++b)
                     ptx::tma_load_3d_hint(sRing + slot * C::kSlotBytes + b * (kBlockN * 128), kv ? tmV : tmK,
-                                          bar(C::kBarFull + slot), b * 64, u.kvh, u.k_row0 + j * kBlockN, keep);
+                                          bar(C::kBarFull + slot), b * 64, u.kvh, u.k_row0 + (u.tile0 + j) * kBlockN,
+                                          keep);
                 ++ring_issued;
                 if (++slot == C::kSlots) {
                     slot = 0;
@@ -226,7 +232,7 @@ __device__ __forceinline__ void run_producer_paged(const CUtensorMap* tmQ, const
             // this lane's page of tile j (the page id is the same for K and V)
             int row = 0;
             if (lane < pages_per_tile) {
-                const int page_idx = min(((j * kBlockN) >> p.page_shift) + lane, last_page);
+                const int page_idx = min((((u.tile0 + j) * kBlockN) >> p.page_shift) + lane, last_page);
                 row = static_cast<int>(static_cast<uint32_t>(table[page_idx]) << p.page_shift);
             }
             for (int kv = 0; kv < 2; ++kv) {
@@ -505,10 +511,87 @@ __device__ __forceinline__ void store_o_rows(const KParams& p, const CUtensorMap
     }
 }
 
+// Epilogue of one warp's rows for a piece of a split unit.  The piece writes
+// its partial result, O / lh in fp32 and the log2-domain LSE of each row,
+// then counts itself on the warp's merge counter of the unit.  The piece
+// that brings the counter to n_chunks (in this launch's epoch) merges the
+// pieces' partials of its 32 rows, O = sum_k 2^(lse_k - M) O_k / W with
+// M = max_k lse_k and W = sum_k 2^(lse_k - M), LSE = M + log2 W, puts O
+// back into its TMEM accumulator and stores it like an unsplit unit.  Every
+// piece of a unit has the same rows in the same warps, so a warp only ever
+// reads partials of its own rows and needs no other warp of its CTA.
 template <int D>
+__device__ __forceinline__ void store_piece(const KParams& p, const CUtensorMap* tmO, uint32_t sStage, uint32_t tO,
+                                            const UnitRec& u, int row_u, int warp_u, float inv_l, float lse2,
+                                            bool valid, int64_t row_idx, int lane, uint32_t epoch, int32_t c_head,
+                                            int32_t c_tok) {
+    // [part][d / 4][kUnitRows][4]: the warp's 32 rows are 512 contiguous bytes per channel quad
+    float4* po = reinterpret_cast<float4*>(p.part_o + static_cast<int64_t>(u.part) * kUnitRows * D) + row_u;
+#pragma unroll
+    for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t ov[32];
+        load_row<32>(tO + 32 * ch, ov);
+#pragma unroll
+        for (int t = 0; t < 8; ++t)
+            po[(ch * 8 + t) * kUnitRows] =
+                make_float4(__uint_as_float(ov[4 * t]) * inv_l, __uint_as_float(ov[4 * t + 1]) * inv_l,
+                            __uint_as_float(ov[4 * t + 2]) * inv_l, __uint_as_float(ov[4 * t + 3]) * inv_l);
+    }
+    p.part_lse[static_cast<int64_t>(u.part) * kUnitRows + row_u] = lse2;
+    __threadfence();
+    __syncwarp();
+    uint32_t count = 0;
+    if (lane == 0) count = count_arrival(p.counters + static_cast<int64_t>(u.group) * kUnitWarps + warp_u, epoch);
+    count = __shfl_sync(0xFFFFFFFFu, count, 0);
+    if (count != static_cast<uint32_t>(u.n_chunks)) return;
+    __threadfence();
+    const int part0 = u.part - u.chunk;
+    const float* pl = p.part_lse + static_cast<int64_t>(part0) * kUnitRows + row_u;
+    float M = -INFINITY;
+    for (int k = 0; k < u.n_chunks; ++k) M = fmaxf(M, __ldcg(pl + k * kUnitRows));
+    float W = 0.f;
+    for (int k = 0; k < u.n_chunks; ++k) {
+        const float lk = __ldcg(pl + k * kUnitRows);
+        W += lk == -INFINITY ? 0.f : ptx::ex2_approx(lk - M);
+    }
+    const float inv_w = W > 0.f ? 1.f / W : 0.f;
+    const float4* src0 = reinterpret_cast<const float4*>(p.part_o + static_cast<int64_t>(part0) * kUnitRows * D) + row_u;
+#pragma unroll 1
+    for (int ch = 0; ch < D / 32; ++ch) {
+        float acc[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+#pragma unroll 1
+        for (int k = 0; k < u.n_chunks; ++k) {
+            const float lk = __ldcg(pl + k * kUnitRows);
+            const float wk = lk == -INFINITY ? 0.f : ptx::ex2_approx(lk - M) * inv_w;
+            const float4* src = src0 + static_cast<int64_t>(k) * (kUnitRows * D / 4) + ch * 8 * kUnitRows;
+            float4 x[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) x[t] = __ldcg(src + t * kUnitRows);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                acc[4 * t] = fmaf(wk, x[t].x, acc[4 * t]);
+                acc[4 * t + 1] = fmaf(wk, x[t].y, acc[4 * t + 1]);
+                acc[4 * t + 2] = fmaf(wk, x[t].z, acc[4 * t + 2]);
+                acc[4 * t + 3] = fmaf(wk, x[t].w, acc[4 * t + 3]);
+            }
+        }
+        uint32_t ov[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(acc[i]);
+        ptx::tmem_st32(tO + 32 * ch, ov);
+    }
+    ptx::tmem_wait_st();
+    store_o_rows<D>(p, tmO, sStage, tO, 1.f, valid, row_idx, lane, c_head, c_tok);
+    if (valid) p.lse[row_idx] = W > 0.f ? (M + log2f(W)) * kLn2 : -INFINITY;
+}
+
+// kPieces: the work list has pieces of split units.
+template <int D, bool kPieces>
 __device__ __forceinline__ void softmax_units(const KParams& p, const CUtensorMap* tmO, int ubeg, int uend,
                                               uint32_t tmem, uint32_t sBar, uint32_t sStage, int warp, int lane,
-                                              volatile int32_t* abort_flag) {
+                                              uint32_t epoch, volatile int32_t* abort_flag) {
     using C = Cfg<D>;
     auto bar = [&](int i) { return sBar + 8u * static_cast<uint32_t>(i); };
     const int mt = (warp - kWarpSoftmax) >> 2;  // M-tile
@@ -533,8 +616,12 @@ __device__ __forceinline__ void softmax_units(const KParams& p, const CUtensorMa
             if (valid) store_zero_row<D>(p, row_idx);
             continue;
         }
-        const int lim = min(u.qlim0 + tok, u.Lk - 1);                 // this row's last visible key
-        const int tile_min_lim = min(u.qlim0 + mt * TPB, u.Lk - 1);  // smallest limit in the M-tile
+        // Key limits relative to the unit's first visited tile (tile0 > 0 for a
+        // later piece of a split unit): this row's last visible key, and the
+        // smallest such limit in the M-tile.
+        const int kofs = u.tile0 * kBlockN;
+        const int lim = min(u.qlim0 + tok, u.Lk - 1) - kofs;
+        const int tile_min_lim = min(u.qlim0 + mt * TPB, u.Lk - 1) - kofs;
         float m = -INFINITY;  // subtraction base, log2 domain
         float l = 0.f;        // running sum of the probabilities (fp32, for LSE)
         float lh = 0.f;       // running sum of the bf16-rounded probabilities PV consumes (normalises O)
@@ -607,6 +694,14 @@ __device__ __forceinline__ void softmax_units(const KParams& p, const CUtensorMa
         // origin of the TMA box of this warp's 32 rows: (channel, head, token)
         const int tok_w = mt * TPB + (quarter * 32) / G;
         const int head_w = (quarter * 32) % G;
+        if constexpr (kPieces) {
+            if (u.part >= 0) {
+                store_piece<D>(p, tmO, sStage, tO, u, mt * kRowsPerTile + r, mt * 4 + quarter, inv_l,
+                               l > 0.f ? m + log2f(l) : -INFINITY, valid, row_idx, lane, epoch, u.kvh * G + head_w,
+                               u.q_tok0 + tok_w);
+                continue;
+            }
+        }
         store_o_rows<D>(p, tmO, sStage, tO, inv_l, valid, row_idx, lane, u.kvh * G + head_w, u.q_tok0 + tok_w);
         if (valid) p.lse[row_idx] = lse_v;
     }
@@ -614,16 +709,19 @@ __device__ __forceinline__ void softmax_units(const KParams& p, const CUtensorMa
 
 // Softmax warpgroup role; lane 0 lets its TMA stores finish before the CTA
 // exits, also when a wait timed out.
-template <int D>
+template <int D, bool kPieces>
 __device__ __forceinline__ void run_softmax(const KParams& p, const CUtensorMap* tmO, int ubeg, int uend,
                                             uint32_t tmem, uint32_t sBar, uint32_t sStage, int warp, int lane,
-                                            volatile int32_t* abort_flag) {
-    softmax_units<D>(p, tmO, ubeg, uend, tmem, sBar, sStage, warp, lane, abort_flag);
+                                            uint32_t epoch, volatile int32_t* abort_flag) {
+    softmax_units<D, kPieces>(p, tmO, ubeg, uend, tmem, sBar, sStage, warp, lane, epoch, abort_flag);
     if (lane == 0) ptx::bulk_wait_all();
     __syncwarp();
 }
 
-template <int D>
+// kPieces selects the build for work lists with pieces of split units; lists
+// without any run a build that carries none of the piece epilogue (a single
+// build measured ~2% slower on unsplit batches).
+template <int D, bool kPieces>
 __global__ void __launch_bounds__(kThreads, 1)
     opattn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                           const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
@@ -638,6 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t sBar = base + C::kBarOff;
     volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(gbase + C::kMiscOff);
     volatile int32_t* abort_flag = reinterpret_cast<volatile int32_t*>(gbase + C::kMiscOff + 4);
+    volatile uint32_t* epoch_slot = reinterpret_cast<volatile uint32_t*>(gbase + C::kMiscOff + 8);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -657,6 +756,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mbar_init(sBar + 8u * C::kBarDrain, 1);
         ptx::mbar_init(sBar + 8u * C::kBarNever, 1);
         *abort_flag = 0;
+        if constexpr (kPieces) *epoch_slot = run_epoch(p.run);
         ptx::fence_mbar_init();
     }
     if (warp == kWarpMma) {
@@ -673,6 +773,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    const uint32_t epoch = kPieces ? *epoch_slot : 0u;
     const int ubeg = p.cta_off[blockIdx.x];
     const int uend = p.cta_off[blockIdx.x + 1];
 
@@ -693,7 +794,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         ptx::setmaxnreg_inc<kRegsSoftmax>();
         const uint32_t sStage = base + C::kStageOff + static_cast<uint32_t>(warp - kWarpSoftmax) * C::kStageBytes;
-        run_softmax<D>(p, &tmO, ubeg, uend, tmem, sBar, sStage, warp, lane, abort_flag);
+        run_softmax<D, kPieces>(p, &tmO, ubeg, uend, tmem, sBar, sStage, warp, lane, epoch, abort_flag);
     }
 
     ptx::tc_fence_before();
@@ -702,6 +803,41 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);
     }
+    if constexpr (kPieces)
+        if (threadIdx.x == 0) run_exit(p.run, epoch);
+}
+
+template <int D, bool kPieces>
+int launch_kernel(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const CUtensorMap& to,
+                  const KParams& kp, int n_cta, cudaStream_t stream) {
+    using C = Cfg<D>;
+    static std::mutex mu;
+    static bool attr_done[128] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    {
+        std::lock_guard<std::mutex> g(mu);
+        if (dev < 0 || dev >= 128 || !attr_done[dev]) {
+            e = cudaFuncSetAttribute(opattn_prefill_kernel<D, kPieces>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     C::kSmemBytes);
+            if (e != cudaSuccess) return e;
+            if (dev >= 0 && dev < 128) attr_done[dev] = true;
+        }
+    }
+    {
+        // The warpgroup register split assumes exactly kLaunchRegs registers
+        // per thread at launch; never launch a build that differs.
+        static std::once_flag once;
+        static int regs = -1;
+        std::call_once(once, [] {
+            cudaFuncAttributes fa;
+            if (cudaFuncGetAttributes(&fa, opattn_prefill_kernel<D, kPieces>) == cudaSuccess) regs = fa.numRegs;
+        });
+        if (regs != kLaunchRegs) return -6;
+    }
+    opattn_prefill_kernel<D, kPieces><<<n_cta, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, to, kp);
+    return cudaGetLastError();
 }
 
 template <int D>
@@ -738,31 +874,6 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     const uint32_t o_tokens = o_tma ? 32u / o_heads : 1u;
     if (!encode_3d(fn, &to, a.o, D, a.Hq, a.total_q, o_heads, o_tokens)) return -7;
 
-    static std::mutex mu;
-    static bool attr_done[128] = {};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    {
-        std::lock_guard<std::mutex> g(mu);
-        if (dev < 0 || dev >= 128 || !attr_done[dev]) {
-            e = cudaFuncSetAttribute(opattn_prefill_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     C::kSmemBytes);
-            if (e != cudaSuccess) return e;
-            if (dev >= 0 && dev < 128) attr_done[dev] = true;
-        }
-    }
-    {
-        // The warpgroup register split assumes exactly kLaunchRegs registers
-        // per thread at launch; never launch a build that differs.
-        static std::once_flag once;
-        static int regs = -1;
-        std::call_once(once, [] {
-            cudaFuncAttributes fa;
-            if (cudaFuncGetAttributes(&fa, opattn_prefill_kernel<D>) == cudaSuccess) regs = fa.numRegs;
-        });
-        if (regs != kLaunchRegs) return -6;
-    }
     KParams kp;
     kp.units = a.units;
     kp.cta_off = a.cta_off;
@@ -778,8 +889,12 @@ int launch_d(const LaunchArgs& a, cudaStream_t stream) {
     kp.max_blocks = a.max_blocks;
     kp.page_shift = page_shift;
     kp.o_tma = o_tma ? 1 : 0;
-    opattn_prefill_kernel<D><<<a.n_cta, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, to, kp);
-    return cudaGetLastError();
+    kp.counters = a.counters;
+    kp.run = a.run;
+    kp.part_lse = a.part_lse;
+    kp.part_o = a.part_o;
+    if (a.part_o) return launch_kernel<D, true>(tq, tk, tv, to, kp, a.n_cta, stream);
+    return launch_kernel<D, false>(tq, tk, tv, to, kp, a.n_cta, stream);
 }
 
 }  // namespace

@@ -282,3 +282,24 @@ def to_paged(x: torch.Tensor, k_lens, layout: PagedLayout, fill: float = 7.0) ->
 
 STANDARD = {"tiny": tiny, "llama3_8b": llama3_8b, "llama3_70b": llama3_70b,
             "bursty": bursty, "chunked": chunked}
+
+
+# --------------------------------------------------------------------------
+# Chunked prefill of few requests over long cached prefixes (split-KV)
+# --------------------------------------------------------------------------
+
+def chunk_long_prefix(seed: int = 0) -> Workload:
+    """One request's 512-token prompt chunk attending to a 16384-token cached prefix (chunked
+    prefill, the step a long prompt takes once its earlier chunks are in the cache); Llama-3-8B
+    heads (Hq 32, Hkv 8, d 128).  Its 64 work units are fewer than the SMs."""
+    return Workload("chunk_1x512_prefix16k", [512], [512 + 16384], 32, 8, 128, 1.0, seed)
+
+
+def chunks_long_prefix(seed: int = 0) -> Workload:
+    """Four requests' 512-token chunks over prefixes drawn uniformly from [8192, 16384]
+    (stream 4); Llama-3-8B heads."""
+    pre = [8192 + p for p in chunk_prefixes(seed, 4, hi=8192)]
+    return Workload("chunks_4x512_prefix8k_16k", [512] * 4, [512 + p for p in pre], 32, 8, 128, 1.0, seed)
+
+
+LONG_PREFIX = {"chunk_long_prefix": chunk_long_prefix, "chunks_long_prefix": chunks_long_prefix}

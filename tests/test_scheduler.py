@@ -2,10 +2,12 @@
 
 The unit records are checked against a brute-force enumeration of which
 (query token, key) pairs the causal mask leaves visible, and the assignment
-against a replay of its rule: (sequence, kv head) pairs gathered in order
+against a replay of its rules: (sequence, kv head) pairs gathered in order
 into groups of at most 48 MB of K/V, units taken group by group and longest
 first within a group, each given to the least-loaded CTA (list scheduling:
-makespan within mean load + largest unit).
+makespan within mean load + largest unit); or, when that makespan is set by
+a few long units, the stream-K cut of all key tiles into one equal stretch
+per CTA, with the units cut by stretch boundaries split into pieces.
 """
 import numpy as np
 import pytest
@@ -37,8 +39,18 @@ CASES = [
 ]
 
 
-@pytest.mark.parametrize("case", CASES)
+SPLIT_CASES = [
+    ([512], [16896], 32, 8, 128, 152),                        # one chunk over a 16K prefix
+    ([512, 512, 300], [9000, 17000, 12000], 32, 8, 128, 152),  # a few chunks over long prefixes
+    ([64, 0, 2000], [40000, 5, 2000], 16, 2, 64, 100),        # G = 8, d = 64, an empty sequence
+    ([5, 3], [3000, 1], 12, 4, 128, 8),                       # G = 3, Lq > Lk rows
+]
+
+
+@pytest.mark.parametrize("case", CASES + SPLIT_CASES)
 def test_units_cover_every_row_once_with_exact_tile_counts(case):
+    """Every (token, kv head) row is in exactly one unit, and the pieces of a split unit
+    cover its key tiles [0, n_tiles) once, in order, with contiguous partial slots."""
     lq, lk, Hq, Hkv, d, n_cta = case
     cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
     cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
@@ -47,6 +59,7 @@ def test_units_cover_every_row_once_with_exact_tile_counts(case):
     tpu = 2 * (128 // G)
     t = unit_table(units)
     covered = np.zeros((int(cu_q[-1]), Hkv), dtype=np.int32)
+    pieces = {}
     for u in range(len(units)):
         s = t["seq"][u]
         L_q, L_k = lq[s], lk[s]
@@ -56,12 +69,35 @@ def test_units_cover_every_row_once_with_exact_tile_counts(case):
         assert t["n_tok"][u] == min(tpu, L_q - tok0)
         assert t["k_row0"][u] == cu_k[s] and t["Lk"][u] == L_k
         assert t["qlim0"][u] == tok0 + delta
-        covered[t["q_tok0"][u]:t["q_tok0"][u] + t["n_tok"][u], t["kvh"][u]] += 1
+        pieces.setdefault((s, t["kvh"][u], tok0), []).append(u)
+    slots, groups = set(), set()
+    for (s, h, tok0), us in pieces.items():
+        L_q, L_k = lq[s], lk[s]
+        n_tok = min(tpu, L_q - tok0)
+        covered[cu_q[s] + tok0:cu_q[s] + tok0 + n_tok, h] += 1
         # brute force: the highest key any token of the unit sees
-        last = max([min(i + delta, L_k - 1) for i in range(tok0, tok0 + t["n_tok"][u])])
+        last = max([min(i + L_k - L_q, L_k - 1) for i in range(tok0, tok0 + n_tok)])
         want_tiles = 0 if last < 0 else last // BN + 1
-        assert t["n_tiles"][u] == want_tiles
+        us = sorted(us, key=lambda u: t["chunk"][u])
+        k = len(us)
+        assert [t["chunk"][u] for u in us] == list(range(k))
+        assert all(t["n_chunks"][u] == k for u in us)
+        tiles = [(t["tile0"][u], t["n_tiles"][u]) for u in us]
+        assert tiles[0][0] == 0 and sum(n for _, n in tiles) == want_tiles
+        assert all(a0 + an == b0 for (a0, an), (b0, _) in zip(tiles, tiles[1:]))
+        if k == 1:
+            assert t["part"][us[0]] == -1 and t["group"][us[0]] == -1
+        else:
+            assert all(n > 0 for _, n in tiles)
+            part0 = t["part"][us[0]]
+            assert [t["part"][u] for u in us] == list(range(part0, part0 + k))
+            assert len({t["group"][u] for u in us}) == 1
+            slots.update(range(part0, part0 + k))
+            groups.add(t["group"][us[0]])
     assert np.all(covered == 1)
+    assert slots == set(range(len(slots))) and groups == set(range(len(groups)))
+    if case in SPLIT_CASES:
+        assert groups, "a batch of few long units is split"
 
 
 GROUP_BYTES = 48 << 20
@@ -104,38 +140,107 @@ def random_cases(n, seed=123):
 
 # The last case's loads span more buckets than the bucket queue takes
 # (1024 CTAs x 70K-tile units), so the scheduler uses its heap there.
-@pytest.mark.parametrize("case", CASES + [(W.chunked().q_lens, W.chunked().k_lens, 32, 8, 128, 152)] +
-                         random_cases(24) + [([512000], [9000000], 1, 1, 64, 1024)])
-def test_group_major_list_assignment(case):
-    lq, lk, Hq, Hkv, d, n_cta = case
-    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
-    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
-    units, offs = pkg.opattn_schedule(cu_q, cu_k, Hq, Hkv, d, n_cta)
-    n = len(units)
-    if n == 0:
-        return
-    G = Hq // Hkv
-    order = expected_order(lq, lk, Hkv, d, G)
-    assert len(order) == n
-    P = len(offs) - 1
-    assert P == min(n_cta, n)
-    assert offs[0] == 0 and offs[-1] == n and np.all(np.diff(offs) >= 1)
-    # replay the greedy list assignment and compare unit by unit
+SPLIT_GAIN = 0.85  # the cut replaces the list schedule below this fraction of its makespan
+PIECE_OVERHEAD = 2
+MIN_STRETCH = 4    # ... and only when a CTA's stretch has at least this many key tiles
+
+
+def list_schedule(order, n_cta):
     import heapq
+    P = min(n_cta, len(order))
     heap = [(0, c) for c in range(P)]
     per_cta = [[] for _ in range(P)]
     for grp, n_tiles, s, h, t0 in order:
         load, c = heapq.heappop(heap)
-        per_cta[c].append((s, h, t0, n_tiles))
+        per_cta[c].append((s, h, t0, n_tiles, 0, -1, -1, 0, 1))
         heapq.heappush(heap, (load + n_tiles + 1, c))
+    return per_cta
+
+
+def stream_k_schedule(order, n_cta):
+    """The cut of all key tiles, units in pair order, into one equal stretch per CTA."""
+    units = sorted(order, key=lambda k: (k[2], k[3], k[4]))  # pair order: sequence, kv head, block
+    total = sum(u[1] for u in units)
+    P = max(1, min(n_cta, total))
+    bound = lambda c: c * total // P  # noqa: E731
+    per_cta = [[] for _ in range(P)]
+    pos, rr, parts, groups = 0, 0, 0, 0
+    for grp, n_tiles, s, h, t0 in units:
+        if n_tiles <= 0:
+            per_cta[rr].append((s, h, t0, 0, 0, -1, -1, 0, 1))
+            rr = (rr + 1) % P
+            continue
+        c = next(c for c in range(P) if bound(c) <= pos < (bound(c + 1) if c + 1 < P else total + 1))
+        pieces, t, end = [], pos, pos + n_tiles
+        while t < end:
+            stop = min(end, bound(c + 1)) if c + 1 < P else end
+            if stop > t:
+                pieces.append((c, t - pos, stop - t))
+            t, c = stop, c + 1
+        k = len(pieces)
+        for i, (cc, a, n) in enumerate(pieces):
+            per_cta[cc].append((s, h, t0, n, a, parts + i if k > 1 else -1, groups if k > 1 else -1, i, k))
+        if k > 1:
+            parts, groups = parts + k, groups + 1
+        pos = end
+    return per_cta
+
+
+def makespan(per_cta):
+    return max(sum(u[3] + 1 + (PIECE_OVERHEAD if u[5] >= 0 else 0) for u in us) for us in per_cta)
+
+
+@pytest.mark.parametrize("case", CASES + [(W.chunked().q_lens, W.chunked().k_lens, 32, 8, 128, 152)] +
+                         random_cases(24) + [([512000], [9000000], 1, 1, 64, 1024)] + SPLIT_CASES)
+def test_group_major_list_assignment(case):
+    """Replays both schedules and the choice between them, and compares unit by unit."""
+    lq, lk, Hq, Hkv, d, n_cta = case
+    cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+    units, offs = pkg.opattn_schedule(cu_q, cu_k, Hq, Hkv, d, n_cta)
+    G = Hq // Hkv
+    order = expected_order(lq, lk, Hkv, d, G)
+    if len(order) == 0:
+        assert len(units) == 0
+        return
+    want = list_schedule(order, n_cta)
+    lpt = makespan(want)
+    total = sum(u[1] + 1 for u in order)
+    tiles = sum(u[1] for u in order)
+    if tiles >= MIN_STRETCH * n_cta and lpt * SPLIT_GAIN > total / n_cta:
+        sk = stream_k_schedule(order, n_cta)
+        if makespan(sk) < SPLIT_GAIN * lpt:
+            want = sk
+    P = len(offs) - 1
+    assert P == len(want)
+    assert offs[0] == 0 and offs[-1] == len(units) and np.all(np.diff(offs) >= 1)
     t = unit_table(units)
     for c in range(P):
-        got = [(int(t["seq"][i]), int(t["kvh"][i]), int(t["q_tok0"][i] - cu_q[t["seq"][i]]), int(t["n_tiles"][i]))
+        got = [(int(t["seq"][i]), int(t["kvh"][i]), int(t["q_tok0"][i] - cu_q[t["seq"][i]]), int(t["n_tiles"][i]),
+                int(t["tile0"][i]), int(t["part"][i]), int(t["group"][i]), int(t["chunk"][i]), int(t["n_chunks"][i]))
                for i in range(offs[c], offs[c + 1])]
-        assert got == per_cta[c], f"CTA {c}"
-    cost = units[:, 6].astype(np.int64) + 1
-    loads = np.array([cost[offs[c]:offs[c + 1]].sum() for c in range(P)])
-    assert loads.max() <= cost.sum() / P + cost.max() + 1e-9
+        assert got == want[c], f"CTA {c}"
+    if (t["part"] < 0).all():  # the list schedule's bound
+        cost = t["n_tiles"].astype(np.int64) + 1
+        loads = np.array([cost[offs[c]:offs[c + 1]].sum() for c in range(P)])
+        assert loads.max() <= cost.sum() / P + cost.max() + 1e-9
+
+
+def test_standard_workloads_are_not_split():
+    for w in [W.llama3_8b(), W.llama3_70b(), W.bursty(), W.chunked(), W.tiny()]:
+        units, _ = pkg.opattn_schedule(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, 152)
+        assert (units[:, pkg.UNIT_FIELDS.index("part")] == -1).all(), w.name
+
+
+def test_small_batches_are_not_split():
+    """Fewer key tiles than 4 per CTA: the list schedule is kept whatever its makespan."""
+    for lq, lk, Hq, Hkv, d in [([300, 45, 129], [300, 45, 129], 16, 4, 128),
+                               ([300, 1, 129, 700], [300, 1, 129, 700], 8, 2, 64),
+                               ([300, 1, 129, 700], [300, 1, 129, 700], 8, 8, 64)]:
+        cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+        cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+        units, _ = pkg.opattn_schedule(cu_q, cu_k, Hq, Hkv, d, 152)
+        assert (units[:, pkg.UNIT_FIELDS.index("part")] == -1).all()
 
 
 def test_groups_keep_each_groups_kv_within_l2():
@@ -155,7 +260,7 @@ def test_capacity_error_reports_the_needed_size():
     lib = pkg.load()
     import ctypes
     n_units, n_used = ctypes.c_int64(0), ctypes.c_int32(0)
-    units = np.zeros((2, 8), dtype=np.int32)
+    units = np.zeros((2, len(pkg.UNIT_FIELDS)), dtype=np.int32)
     offs = np.zeros(8, dtype=np.int32)
     st = lib.opattn_schedule(cu.ctypes.data_as(ctypes.c_void_p), cu.ctypes.data_as(ctypes.c_void_p), 1, 8, 2, 128, 4,
                              units.ctypes.data_as(ctypes.c_void_p), 2, offs.ctypes.data_as(ctypes.c_void_p),
