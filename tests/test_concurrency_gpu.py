@@ -26,6 +26,7 @@ def built():
 
 PREFILL = W.Workload("det_prefill", [300, 1000, 45], [300, 1500, 45], 32, 8, 128, 1.0, 21)
 DECODE = W.Workload("det_decode", [1, 2, 1], [30000, 9000, 640], 16, 2, 128, 1.0, 22)
+SPLIT = W.Workload("det_split", [200], [20000], 16, 4, 128, 1.0, 23)  # prefill units cut into pieces
 
 
 def outputs(w):
@@ -34,13 +35,14 @@ def outputs(w):
     return o, lse
 
 
-@pytest.mark.parametrize("w,decode", [(PREFILL, False), (DECODE, True)], ids=["prefill", "decode"])
+@pytest.mark.parametrize("w,decode", [(PREFILL, False), (DECODE, True), (SPLIT, False)],
+                         ids=["prefill", "decode", "prefill_split"])
 def test_repeated_runs_are_bitwise_identical(w, decode):
     q, k, v = W.make_inputs(w, "cuda")
     runs = []
     with pkg.Plan(w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, decode=decode) as plan:
-        if decode:
-            assert plan.n_units > w.n_seq * w.Hkv        # split key ranges, merged in-kernel
+        if decode or w is SPLIT:
+            assert plan.n_units > w.n_seq * w.Hkv * (1 if decode else 4)  # split key ranges, merged in-kernel
         for _ in range(3):
             o, lse = outputs(w)
             plan.run(q, k, v, o, lse, w.scale)
@@ -52,10 +54,11 @@ def test_repeated_runs_are_bitwise_identical(w, decode):
 
 
 def test_concurrent_host_threads_match_a_lone_call():
-    inputs = {name: W.make_inputs(w, "cuda") for name, w in (("prefill", PREFILL), ("decode", DECODE))}
-    calls = {"prefill": pkg.opattn_prefill, "decode": pkg.opattn_decode}
+    cases = (("prefill", PREFILL), ("decode", DECODE), ("split", SPLIT))
+    inputs = {name: W.make_inputs(w, "cuda") for name, w in cases}
+    calls = {"prefill": pkg.opattn_prefill, "decode": pkg.opattn_decode, "split": pkg.opattn_prefill}
     ref = {}
-    for name, w in (("prefill", PREFILL), ("decode", DECODE)):
+    for name, w in cases:
         o, lse = outputs(w)
         calls[name](*inputs[name], o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale)
         torch.cuda.synchronize()
@@ -67,7 +70,7 @@ def test_concurrent_host_threads_match_a_lone_call():
             stream = torch.cuda.Stream()
             with torch.cuda.stream(stream):
                 for it in range(6):
-                    name, w = (("prefill", PREFILL), ("decode", DECODE))[(tid + it) % 2]
+                    name, w = cases[(tid + it) % 3]
                     o, lse = outputs(w)
                     calls[name](*inputs[name], o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale,
                                 stream)
