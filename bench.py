@@ -291,7 +291,7 @@ def run_reference(args, w):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded N(0,1) bf16 inputs; counter-based generator)",
-        "config": dict(w.describe(), sample="random (token, head) rows per step"),
+        "config": bench_config(w, args.gpus),
         "tokens_per_s": tokens_per_s,
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
@@ -553,8 +553,7 @@ def run_ours(args, w):
             "warmup": args.warmup, "ms_per_step": elapsed_max / args.steps * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded N(0,1) bf16 q/k/v from a counter-based generator)",
-            "config": dict(w.describe(), parallelism=f"replicas{world}" if world > 1 else "single_gpu",
-                           l2="inputs larger than L2 (q+k+v+o of the workload exceed the 129 MB L2)"),
+            "config": bench_config(w, world),
             "tokens_per_s": value * 1e12 / (flops / w.total_q),
             "pct_bf16_peak": value / peak,
             "pct_bf16_peak_sustained": value / peak_sus,
@@ -579,6 +578,12 @@ def run_ours(args, w):
         dist.barrier()
         dist.destroy_process_group()
     return 0
+
+
+def bench_config(w, world: int) -> dict:
+    """The workload description both arms print as `config` (the same dict, so the two lines compare)."""
+    return dict(w.describe(), parallelism=f"replicas{world}" if world > 1 else "single_gpu",
+                l2="inputs larger than L2 (q+k+v+o of the workload exceed the 129 MB L2)")
 
 
 def is_decode(w) -> bool:

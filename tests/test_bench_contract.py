@@ -26,6 +26,11 @@ def test_reference_arm_prints_one_contract_line():
     assert j["value"] > 0 and j["ms_per_step"] > 0 and j["higher_is_better"] is True
     assert j["unit"] == "TFLOP/s" and j["dtype"] == "f64"
     assert j["config"]["workload"].startswith("tiny")
+    # the same config dict as the GPU arm prints, so that the two lines compare
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_13499_gb300 import workloads as W
+    assert j["config"] == json.loads(json.dumps(bench.bench_config(W.tiny(), 1)))
     assert j["e2e"] == {"value": j["value"], "unit": j["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     cb = j["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == j["value"] and cb["cores"] >= 1 and cb["sample"]
