@@ -86,8 +86,11 @@ OPATTN_API const char *opattn_status_string(int32_t status);
  * are split: 129 fp32 per row of a piece at d = 128) is allocated with
  * cudaMallocFromPoolAsync from a memory pool the library creates per device
  * and freed on `stream`; the pool keeps up to 64 MB of freed scratch mapped
- * between calls.  Returns OPATTN_OK with no
- * device work when total_q == 0.  `scale` must be finite and > 0 (usually
+ * between calls.  The scheduler's host working arrays are kept per calling
+ * thread and reused by its next call (they grow to the largest batch the
+ * thread has scheduled, about 120 bytes per work unit), so that a call
+ * allocates no host memory once the thread has seen a batch as large.
+ * Returns OPATTN_OK with no device work when total_q == 0.  `scale` must be finite and > 0 (usually
  * 1 / sqrt(d)).  Device-side wait timeouts are not reported here; use
  * opattn_prefill_checked to observe them.
  */

@@ -98,27 +98,40 @@ constexpr int64_t kL2GroupBytes = 48ll << 20;
 // pairs.  Batches whose buckets would take more than kMaxBucketWords words
 // use a heap of (load, index) pairs instead.
 // The units are taken in the order order[0], order[1], ... (indices into `all`).
+// The working arrays are kept per host thread and reused, so that a call
+// allocates (and page-faults in) nothing once the thread has scheduled a
+// batch as large.
 template <class U, class CostFn>
 void list_pack(const std::vector<U>& all, const std::vector<uint32_t>& order, int32_t max_ctas, CostFn cost,
                std::vector<U>* units, std::vector<int32_t>* cta_off, int32_t* n_cta_out) {
     auto ordered = [&](int64_t i) -> const U& { return all[order[static_cast<size_t>(i)]]; };
     const int64_t n = static_cast<int64_t>(order.size());
-    units->clear();
     cta_off->clear();
     *n_cta_out = 0;
-    if (n == 0) return;
+    if (n == 0) {
+        units->clear();
+        return;
+    }
     const int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(std::max<int32_t>(max_ctas, 1), n));
-    std::vector<int32_t> owner(static_cast<size_t>(n));
-    std::vector<int32_t> per_cta(static_cast<size_t>(n_cta), 0);
+    thread_local std::vector<int32_t> owner, per_cta, costs, count, fill;
+    thread_local std::vector<uint64_t> bits;
+    thread_local std::vector<int64_t> load;
+    owner.resize(static_cast<size_t>(n));
+    costs.resize(static_cast<size_t>(n));
+    per_cta.assign(static_cast<size_t>(n_cta), 0);
     int64_t max_cost = 1;
-    for (int64_t i = 0; i < n; ++i) max_cost = std::max<int64_t>(max_cost, cost(ordered(i)));
+    for (int64_t i = 0; i < n; ++i) {
+        const int64_t c = cost(ordered(i));
+        costs[static_cast<size_t>(i)] = static_cast<int32_t>(c);
+        max_cost = std::max<int64_t>(max_cost, c);
+    }
     const size_t words = (static_cast<size_t>(n_cta) + 63) / 64;
     constexpr size_t kMaxBucketWords = size_t{1} << 20;
     const size_t n_buckets = static_cast<size_t>(max_cost) + 1;
     if (n_buckets * words <= kMaxBucketWords) {
-        std::vector<uint64_t> bits(n_buckets * words, 0);
-        std::vector<int32_t> count(n_buckets, 0);
-        std::vector<int64_t> load(static_cast<size_t>(n_cta), 0);
+        bits.assign(n_buckets * words, 0);
+        count.assign(n_buckets, 0);
+        load.assign(static_cast<size_t>(n_cta), 0);
         for (int32_t c = 0; c < n_cta; ++c) bits[static_cast<size_t>(c) >> 6] |= uint64_t{1} << (c & 63);
         count[0] = n_cta;
         int64_t least = 0;  // least load of any CTA
@@ -136,9 +149,11 @@ void list_pack(const std::vector<U>& all, const std::vector<uint32_t>& order, in
             --count[b];
             owner[static_cast<size_t>(i)] = c;
             ++per_cta[static_cast<size_t>(c)];
-            const int64_t nl = load[static_cast<size_t>(c)] + cost(ordered(i));
+            const int64_t nl = load[static_cast<size_t>(c)] + costs[static_cast<size_t>(i)];
             load[static_cast<size_t>(c)] = nl;
-            const size_t nb = static_cast<size_t>(nl % static_cast<int64_t>(n_buckets));
+            // c came from bucket b (load `least`) and costs are below n_buckets
+            size_t nb = b + static_cast<size_t>(costs[static_cast<size_t>(i)]);
+            if (nb >= n_buckets) nb -= n_buckets;
             bits[nb * words + (static_cast<size_t>(c) >> 6)] |= uint64_t{1} << (c & 63);
             ++count[nb];
         }
@@ -151,14 +166,14 @@ void list_pack(const std::vector<U>& all, const std::vector<uint32_t>& order, in
             heap.pop();
             owner[static_cast<size_t>(i)] = sl.second;
             ++per_cta[static_cast<size_t>(sl.second)];
-            sl.first += cost(ordered(i));
+            sl.first += costs[static_cast<size_t>(i)];
             heap.push(sl);
         }
     }
     cta_off->assign(static_cast<size_t>(n_cta) + 1, 0);
     for (int32_t c = 0; c < n_cta; ++c)
         (*cta_off)[static_cast<size_t>(c) + 1] = (*cta_off)[static_cast<size_t>(c)] + per_cta[static_cast<size_t>(c)];
-    std::vector<int32_t> fill(cta_off->begin(), cta_off->end() - 1);
+    fill.assign(cta_off->begin(), cta_off->end() - 1);
     units->resize(static_cast<size_t>(n));
     for (int64_t i = 0; i < n; ++i) {
         const int32_t c = owner[static_cast<size_t>(i)];
@@ -284,16 +299,22 @@ void split_if_faster(const std::vector<UnitRec>& all, int32_t max_ctas, Schedule
 // K/V tile comes from HBM about once; across the whole list the greedy
 // assignment keeps the makespan within mean load + largest unit.  The
 // longest-first order within a group is a stable counting sort on the tile
-// count (O(units + tiles) per group).
+// count (O(units + tiles) per group).  The working arrays are kept per host
+// thread and reused (see list_pack).
 void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g, int32_t max_ctas, Schedule* out,
                     bool allow_split = true) {
     const int32_t tpu = 2 * g.TPB;
     int64_t n_units = 0;
     for (int32_t s = 0; s < g.n_seq; ++s) n_units += (static_cast<int64_t>(cu_q[s + 1] - cu_q[s]) + tpu - 1) / tpu;
     n_units *= g.Hkv;
-    std::vector<UnitRec> all(static_cast<size_t>(n_units));
-    std::vector<size_t> group_start;  // index in `all` of each group's first unit
-    std::vector<int32_t> group_max;   // most key tiles of a unit in the group
+    thread_local std::vector<UnitRec> all;
+    thread_local std::vector<size_t> group_start;  // index in `all` of each group's first unit
+    thread_local std::vector<int32_t> group_max;   // most key tiles of a unit in the group
+    thread_local std::vector<uint32_t> order;
+    thread_local std::vector<size_t> slot;
+    all.resize(static_cast<size_t>(n_units));
+    group_start.clear();
+    group_max.clear();
     int64_t group_bytes = 0;
     const int64_t pair_row_bytes = 2 * static_cast<int64_t>(g.d) * 2;  // K and V, bf16
     size_t n = 0;
@@ -344,8 +365,7 @@ void build_schedule(const int32_t* cu_q, const int32_t* cu_k, const Geometry& g,
         n = first + static_cast<size_t>(g.Hkv) * per_head;
     }
     // group by group, longest first within a group (stable counting sort of indices)
-    std::vector<uint32_t> order(all.size());
-    std::vector<size_t> slot;
+    order.resize(all.size());
     group_start.push_back(all.size());
     for (size_t gi = 0; gi + 1 < group_start.size(); ++gi) {
         const size_t b = group_start[gi], e = group_start[gi + 1];
@@ -647,7 +667,9 @@ opattn_status prefill_impl(const void* q, const void* k, const void* v, void* o,
     const int sms = device_sm_count();
     if (sms <= 0) return OPATTN_ERR_CUDA;
 
-    Schedule sch;
+    // Reused by the thread's next call: the list is copied into the staging
+    // buffer below before this call returns.
+    thread_local Schedule sch;
     build_schedule(cu_q, cu_k, g, sms, &sch);
     log_schedule("prefill", sch.units, sch.cta_off, prefill_cost, us_since(t_entry));
     const WorkLayout w = work_layout(sch, g.d);
@@ -1284,7 +1306,7 @@ opattn_status opattn_schedule(const int32_t* cu_seqlens_q, const int32_t* cu_seq
     Geometry g;
     opattn_status st = check_geometry(cu_seqlens_q, cu_seqlens_k, n_seq, Hq, Hkv, d, &g);
     if (st != OPATTN_OK) return st;
-    Schedule sch;
+    thread_local Schedule sch;  // copied out below; reused by the thread's next call
     const Clock::time_point t0 = Clock::now();
     build_schedule(cu_seqlens_q, cu_seqlens_k, g, n_ctas, &sch);
     log_schedule("prefill schedule", sch.units, sch.cta_off, prefill_cost, us_since(t0));
