@@ -405,10 +405,15 @@ WorkLayout work_layout(const Schedule& s, int32_t d) {
     w.bytes = w.off_part_o + static_cast<size_t>(s.n_parts) * kUnitRows * static_cast<size_t>(d) * sizeof(float);
     return w;
 }
+// Writes each byte of the upload once: the offsets, the units and zeros in
+// the two alignment gaps.
 void pack_upload(const Schedule& s, const WorkLayout& w, uint8_t* dst) {
-    std::memset(dst, 0, w.upload_bytes);
-    std::memcpy(dst, s.cta_off.data(), s.cta_off.size() * sizeof(int32_t));
+    const size_t off_bytes = s.cta_off.size() * sizeof(int32_t);
+    const size_t end_units = w.off_units + s.units.size() * sizeof(UnitRec);
+    std::memcpy(dst, s.cta_off.data(), off_bytes);
+    std::memset(dst + off_bytes, 0, w.off_units - off_bytes);
     std::memcpy(dst + w.off_units, s.units.data(), s.units.size() * sizeof(UnitRec));
+    std::memset(dst + end_units, 0, w.upload_bytes - end_units);
 }
 
 // ------------------------------------------------------ OPATTN_LOG=1
@@ -1017,9 +1022,12 @@ DecodeLayout decode_layout(const DecodeSchedule& s) {
     return w;
 }
 void pack_decode_upload(const DecodeSchedule& s, const DecodeLayout& w, uint8_t* dst) {
-    std::memset(dst, 0, w.upload_bytes);
-    std::memcpy(dst, s.cta_off.data(), s.cta_off.size() * sizeof(int32_t));
+    const size_t off_bytes = s.cta_off.size() * sizeof(int32_t);
+    const size_t end_units = w.off_units + s.units.size() * sizeof(DecUnit);
+    std::memcpy(dst, s.cta_off.data(), off_bytes);
+    std::memset(dst + off_bytes, 0, w.off_units - off_bytes);
     std::memcpy(dst + w.off_units, s.units.data(), s.units.size() * sizeof(DecUnit));
+    std::memset(dst + end_units, 0, w.upload_bytes - end_units);
 }
 DecodeLaunchArgs make_decode_args(const void* q, const void* k, const void* v, void* o, float* lse,
                                   const Geometry& g, float scale, uint8_t* work, const DecodeLayout& w,
