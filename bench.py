@@ -416,14 +416,14 @@ def run_ours(args, w):
 
     # End to end through the one-shot C-ABI call with pinned host buffers.  Every
     # step copies its inputs host -> device, runs the call and copies O and LSE
-    # back, all inside the timed region.  Two device buffer sets and separate
+    # back, all inside the timed region.  Three device buffer sets and separate
     # copy streams let step i + 1's input copy and step i - 1's output copy run
     # while step i computes, as a serving loop that stages the next batch would.
-    # As many steps as the device-timed region (unless --e2e-steps asks for
-    # fewer), so that the pipeline's fill (the first step's input copy) and
-    # drain (the last step's output copy) weigh as little as they do in a
-    # serving loop.
-    e2e_steps = max(3, min(args.steps, args.e2e_steps if args.e2e_steps > 0 else args.steps))
+    # As many steps as the device-timed region and at least 100 (unless
+    # --e2e-steps sets the count), so that the pipeline's fill (the first
+    # step's input copy) and drain (the last step's output copy) weigh as
+    # little as they do in a serving loop.
+    e2e_steps = max(3, args.e2e_steps) if args.e2e_steps > 0 else max(args.steps, 100)
     hq = q.cpu().pin_memory()
     hk = k.cpu().pin_memory()
     hv = v.cpu().pin_memory()
@@ -629,7 +629,7 @@ def main(argv=None):
                          "chunks_long_prefix | decode_llama3_70b | "
                          "decode_llama3_8b | decode_spec4_llama3_70b | decode_llama3_70b_paged16")
     ap.add_argument("--e2e-steps", type=int, default=0,
-                    help="steps of the end-to-end measurement (default 0: as many as --steps)")
+                    help="steps of the end-to-end measurement (default 0: as many as --steps, at least 100)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--sustained-seconds", type=float, default=3.0,
                     help="duration of the back-to-back 'sustained' measurement (0: skip)")
