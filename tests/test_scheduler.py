@@ -304,3 +304,23 @@ def test_opattn_log_prints_work_list_statistics():
     env["OPATTN_LOG"] = "0"
     r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, check=True)
     assert "opattn:" not in r.stderr
+
+
+def test_repeated_schedules_on_one_thread_are_identical():
+    """The scheduler keeps its working arrays per host thread and reuses them: a list built after
+    larger and smaller ones (arrays grown, then partly reused) must equal the one built first."""
+    shapes = [
+        (W.llama3_8b().q_lens, W.llama3_8b().k_lens, 32, 8, 128, 152),
+        (W.bursty().q_lens, W.bursty().k_lens, 32, 8, 128, 152),   # larger: the arrays grow
+        ([1, 17, 64], [1, 17, 64], 4, 2, 64, 152),                 # smaller: stale tails remain
+        ([512], [16896], 32, 8, 128, 152),                         # the split-KV cut
+    ]
+    def sched(shape):
+        lq, lk, Hq, Hkv, d, n_cta = shape
+        cu_q = np.concatenate([[0], np.cumsum(lq)]).astype(np.int32)
+        cu_k = np.concatenate([[0], np.cumsum(lk)]).astype(np.int32)
+        return pkg.opattn_schedule(cu_q, cu_k, Hq, Hkv, d, n_cta)
+    first = [sched(s) for s in shapes]
+    for s, (u0, o0) in reversed(list(zip(shapes, first))):
+        u1, o1 = sched(s)
+        assert np.array_equal(u0, u1) and np.array_equal(o0, o1)
