@@ -90,6 +90,10 @@ OPATTN_API const char *opattn_status_string(int32_t status);
  * thread and reused by its next call (they grow to the largest batch the
  * thread has scheduled, about 120 bytes per work unit), so that a call
  * allocates no host memory once the thread has seen a batch as large.
+ * The call does not wait for the GPU, except when the host runs 32 calls
+ * ahead of it: the work lists are staged in a pool of at most 32 pinned
+ * buffers, and a call that finds all of them still queued for upload waits
+ * for the oldest upload instead of pinning more memory.
  * Returns OPATTN_OK with no device work when total_q == 0.  `scale` must be finite and > 0 (usually
  * 1 / sqrt(d)).  Device-side wait timeouts are not reported here; use
  * opattn_prefill_checked to observe them.

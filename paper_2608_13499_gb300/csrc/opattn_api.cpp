@@ -462,29 +462,46 @@ int64_t prefill_cost(const UnitRec& u) { return u.n_tiles + 1; }
 // ---------------------------------------------------- pinned staging pool
 // The work list is built in mapped pinned memory and read from there by the
 // upload kernel (opattn_upload.cu); a staging buffer is reused only after
-// the event recorded behind that read has completed, so no call ever blocks
-// on the GPU.  Where the memory cannot be mapped, an asynchronous copy
-// moves it instead.
+// the event recorded behind that read has completed.  Where the memory
+// cannot be mapped, an asynchronous copy moves it instead.  The pool grows
+// while every buffer is in flight, up to kMaxStaging buffers; beyond that a
+// call waits for the upload of the oldest buffer (the host is then that many
+// calls ahead of the GPU) instead of pinning more memory.  A call needing a
+// larger buffer than any free one still gets a new one.
 struct Staging {
     void* host = nullptr;
     void* dev = nullptr;  // device address of the mapped buffer, or null
     size_t cap = 0;
     cudaEvent_t done = nullptr;
     bool busy = false;
+    uint64_t seq = 0;     // release order: the smallest is the oldest upload
 };
+constexpr size_t kMaxStaging = 32;
 std::mutex g_stage_mu;
 std::vector<Staging*> g_stage_pool;
+uint64_t g_stage_seq = 0;
 
 Staging* staging_acquire(size_t bytes) {
-    std::lock_guard<std::mutex> lk(g_stage_mu);
-    for (Staging* s : g_stage_pool) {
-        if (s->busy || s->cap < bytes) continue;
-        if (cudaEventQuery(s->done) != cudaSuccess) {
+    Staging* oldest = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_stage_mu);
+        for (Staging* s : g_stage_pool) {
+            if (s->busy || s->cap < bytes) continue;
+            if (cudaEventQuery(s->done) == cudaSuccess) {
+                s->busy = true;
+                return s;
+            }
             (void)cudaGetLastError();  // cudaErrorNotReady is not an error here
-            continue;
+            if (!oldest || s->seq < oldest->seq) oldest = s;
         }
-        s->busy = true;
-        return s;
+        if (oldest && g_stage_pool.size() >= kMaxStaging)
+            oldest->busy = true;
+        else
+            oldest = nullptr;
+    }
+    if (oldest) {
+        if (cudaEventSynchronize(oldest->done) != cudaSuccess) (void)cudaGetLastError();
+        return oldest;
     }
     Staging* s = new Staging;
     size_t cap = 4096;
@@ -508,12 +525,14 @@ Staging* staging_acquire(size_t bytes) {
     }
     s->cap = cap;
     s->busy = true;
+    std::lock_guard<std::mutex> lk(g_stage_mu);
     g_stage_pool.push_back(s);
     return s;
 }
 void staging_release(Staging* s, cudaStream_t stream) {
     std::lock_guard<std::mutex> lk(g_stage_mu);
     cudaEventRecord(s->done, stream);
+    s->seq = ++g_stage_seq;
     s->busy = false;
 }
 // Moves the first `bytes` of a staged work list to `dst` and zeroes the

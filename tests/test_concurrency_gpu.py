@@ -88,3 +88,23 @@ def test_concurrent_host_threads_match_a_lone_call():
         t.join(timeout=300)
     assert not any(t.is_alive() for t in threads)
     assert not errors, errors
+
+
+def test_calls_queued_far_ahead_of_the_gpu_are_correct():
+    """48 one-shot calls queued behind a kernel that keeps the GPU busy: the host runs more calls
+    ahead than the staging pool holds buffers (32), so later calls wait for the oldest work-list
+    upload and reuse its buffer.  Every call's output must equal a lone call's."""
+    w = PREFILL
+    q, k, v = W.make_inputs(w, "cuda")
+    o_ref, l_ref = outputs(w)
+    pkg.opattn_prefill(q, k, v, o_ref, l_ref, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale)
+    torch.cuda.synchronize()
+    outs = [outputs(w) for _ in range(48)]
+    torch.cuda.synchronize()
+    torch.cuda._sleep(400_000_000)  # ~0.2 s of GPU time ahead of the calls
+    for o, lse in outs:
+        pkg.opattn_prefill(q, k, v, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale)
+    torch.cuda.synchronize()
+    for i, (o, lse) in enumerate(outs):
+        assert torch.equal(o.view(torch.int16), o_ref.view(torch.int16)), f"call {i}: O differs"
+        assert torch.equal(lse.view(torch.int32), l_ref.view(torch.int32)), f"call {i}: LSE differs"
