@@ -10,7 +10,6 @@ every work unit, both M-tiles, every warp's first and last accumulator row,
 with every output element checked for having been written.
 """
 import math
-
 import os
 
 import numpy as np
