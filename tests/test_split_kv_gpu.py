@@ -186,3 +186,31 @@ def test_noalloc_runs_the_unsplit_schedule_within_tolerance():
     pkg.opattn_prefill_noalloc(q, k, v, o, lse, w.cu_q, w.cu_k, w.n_seq, w.Hq, w.Hkv, w.d, w.scale)
     torch.cuda.synchronize()
     check(o, lse, o_ref, lse_ref, "no-alloc")
+
+
+def random_split_case(i):
+    """Seeded random chunked-prefill batch that the scheduler cuts into pieces on a 152-SM GPU:
+    1-4 chunks of 1-300 queries over 8K-40K-key prefixes, G in {1, 2, 3, 4, 8, 16}, d in {64, 128},
+    2 or 4 kv heads.  Draws that the list schedule would keep whole are drawn again."""
+    rng = np.random.default_rng(7000 + i)
+    while True:
+        n = int(rng.integers(1, 5))
+        G = int(rng.choice([1, 2, 3, 4, 8, 16]))
+        Hkv = int(rng.choice([2, 4]))
+        d = int(rng.choice([64, 128]))
+        lq = [int(x) for x in rng.integers(1, 301, n)]
+        lk = [q + int(p) for q, p in zip(lq, rng.integers(8000, 40001, n))]
+        w = custom(f"rand_split_{i}", lq, lk, G * Hkv, Hkv, d, seed=7000 + i)
+        if n_pieces(w, 152) > 0:
+            return w
+
+
+@pytest.mark.parametrize("i", range(10))
+def test_random_split_batches_every_element(i):
+    w = random_split_case(i)
+    if n_pieces(w) == 0:
+        pytest.skip("this batch is not split on this GPU")
+    q, k, v = W.make_inputs(w, "cuda")
+    o, lse = run_gpu(w, q, k, v)
+    o_ref, lse_ref = reference(w, q, k, v)
+    check(o, lse, o_ref, lse_ref, w.name)
