@@ -286,3 +286,22 @@ def test_no_keys_at_all():
     torch.cuda.synchronize()
     assert torch.all(o == 0).item()
     assert torch.all(lse == -math.inf).item()
+
+
+def test_million_token_batch_sampled_rows():
+    """A batch of 2^20 query tokens (256 prompts of 4096, Hq 8, Hkv 2: 32768 work units, q and o
+    2 GB each) against the oracle on 4096 random rows plus every head of the batch's first and
+    last 64 tokens, where packed row indices and TMA coordinates are largest."""
+    w = custom("million", [4096] * 256, [4096] * 256, 8, 2, 128, seed=13)
+    q, k, v = W.make_inputs(w, "cuda")
+    o, lse = run_gpu(w, q, k, v)
+    assert not torch.isnan(o).any().item() and not torch.isnan(lse).any().item()
+    rng = np.random.default_rng(13)
+    edge = np.concatenate([np.arange(64), np.arange(w.total_q - 64, w.total_q)])
+    tok = np.concatenate([rng.integers(0, w.total_q, 4096), np.repeat(edge, w.Hq)]).astype(np.int64)
+    hd = np.concatenate([rng.integers(0, w.Hq, 4096), np.tile(np.arange(w.Hq), len(edge))]).astype(np.int32)
+    o_ref, lse_ref = oracle.attention_rows(q.cpu(), k.cpu(), v.cpu(), w.cu_q, w.cu_k, w.Hq, w.Hkv, w.d, w.scale,
+                                           tok, hd)
+    t_idx = torch.from_numpy(tok)
+    h_idx = torch.from_numpy(hd.astype(np.int64))
+    check(o.cpu()[t_idx, h_idx], lse.cpu()[t_idx, h_idx], o_ref, lse_ref, f"{w.name} ({len(tok)} rows)")
